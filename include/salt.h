@@ -1,0 +1,264 @@
+/*
+ * salt.h - C ABI of the SALT serving hot path on GB300 (sm_103a).
+ *
+ * SALT ("Pin Once, Swap Light", Section "Multi-Tenant Serving") serves a
+ * request with W_final = W_base + gamma * Wbar + delta_i: a high-rank domain
+ * centroid Wbar = A_c B_c stays pinned in device memory, an ultra-low-rank
+ * (r <= 2) user residual delta_i = a_u b_u is swapped in on demand
+ * (Section "The Centroid-Residual Decomposition").  This library evaluates
+ * the LoRA part of that composition for every token of a heterogeneous
+ * batch, in place:
+ *
+ *     y[t, :] += s_c(d) * (x[t, :] A_c(d)) B_c(d) + s_u(u) * (x[t, :] a_u(u)) b_u(u)
+ *
+ * where d is the token's domain (centroid) id and u its residual slot id,
+ * y already holds x W_base, and an id of -1 drops its term.  s_c carries
+ * gamma (and any LoRA alpha/r the caller folds in); s_u the residual's.
+ *
+ * Conventions
+ *  - Math is in row vectors.  A factor is stored transposed: At[k][i] with
+ *    i over d_in (PEFT's lora_A.weight); B[k][j] with j over d_out
+ *    (PEFT's lora_B.weight transposed).  All factors and activations are
+ *    bf16, row-major, passed as raw bit patterns (uint16).
+ *  - A "layer" is one adapted weight matrix (one projection of one
+ *    transformer layer); the context's layer table lists their shapes.
+ *  - Streams are cudaStream_t values passed as void*; NULL is the legacy
+ *    default stream.  Device pointers are CUDA device addresses of the
+ *    context's device; host pointers are ordinary host addresses.
+ *  - Every call returns a salt_status; no C++ exception crosses this ABI.
+ *    On failure salt_last_error(ctx) holds a one-line message.  A context
+ *    is not thread-safe: serialise calls on one context.
+ *  - Calls marked "asynchronous" enqueue work and return without waiting
+ *    for the device; their device-side faults in the ids are reported by
+ *    salt_get_device_error.
+ */
+#ifndef SALT_H
+#define SALT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SALT_ABI_VERSION 1
+
+/* Library limits. */
+#define SALT_MAX_TOKENS 16384        /* tokens per segments build */
+#define SALT_MAX_CENTROID_RANK 64    /* rc_max */
+#define SALT_MAX_RESIDUAL_RANK 16    /* r_max (16 covers the rank-16 LoRA comparison) */
+#define SALT_MAX_GROUP 8             /* projections per grouped apply */
+#define SALT_BLOB_HEADER_BYTES 256
+#define SALT_BLOB_MAGIC 0x3153455254414C53ULL /* "SALTRES1" little-endian */
+
+typedef void *salt_stream_t;
+typedef struct salt_ctx salt_ctx;
+typedef struct salt_segments salt_segments;
+
+typedef enum salt_status {
+    SALT_OK = 0,
+    SALT_ERR_INVALID_ARG = 1,        /* NULL pointer, bad size, bad config */
+    SALT_ERR_OOM = 2,                /* device or pinned-host allocation failed */
+    SALT_ERR_NOT_PINNED_HOST = 3,    /* residual blob is not page-locked host memory */
+    SALT_ERR_DOMAIN_NOT_PINNED = 4,  /* a token names a domain with no pinned centroid */
+    SALT_ERR_SLOT_RANGE = 5,         /* slot id outside [-1, n_slots) */
+    SALT_ERR_RANK = 6,               /* rank above the context's limit, or zero */
+    SALT_ERR_LAYER_RANGE = 7,        /* layer index outside the layer table */
+    SALT_ERR_ALIGN = 8,              /* x / y not 16-byte aligned */
+    SALT_ERR_BAD_BLOB = 9,           /* wrong magic, version, layer count or layout hash */
+    SALT_ERR_DEVICE_IDS = 10,        /* device-side id check failed (see salt_get_device_error) */
+    SALT_ERR_TIMEOUT = 11,           /* reserved: a bounded device wait gave up */
+    SALT_ERR_CUDA = 12,              /* a CUDA runtime call failed */
+    SALT_ERR_SLOT_EMPTY = 13,        /* a token names a slot that was never loaded */
+    SALT_ERR_TOO_MANY_TOKENS = 14,   /* n_tokens above the context's max_tokens */
+    SALT_ERR_DOMAIN_RANGE = 15,      /* domain id outside [-1, n_domains) */
+    SALT_ERR_STALE_SEGMENTS = 16,    /* a slot the segments read was reloaded after the build */
+    SALT_ERR_NOT_BUILT = 17          /* segments object was never built */
+} salt_status;
+
+/* Bits of the device error word (salt_get_device_error). */
+#define SALT_DEVERR_DOMAIN_RANGE 0x1u
+#define SALT_DEVERR_DOMAIN_NOT_PINNED 0x2u
+#define SALT_DEVERR_SLOT_RANGE 0x4u
+#define SALT_DEVERR_SLOT_EMPTY 0x8u
+#define SALT_DEVERR_RANK 0x10u
+
+/*
+ * Context configuration.  d_in / d_out are host arrays of n_layers entries,
+ * each a positive multiple of 8 (16-byte rows).  rc_max <=
+ * SALT_MAX_CENTROID_RANK, 1 <= r_max <= SALT_MAX_RESIDUAL_RANK,
+ * rc_max + r_max <= 128, 1 <= max_tokens <= SALT_MAX_TOKENS.
+ */
+typedef struct salt_config {
+    int32_t n_layers;
+    const int32_t *d_in;
+    const int32_t *d_out;
+    int32_t n_domains;   /* centroid table size */
+    int32_t rc_max;      /* largest centroid rank to be pinned */
+    int32_t n_slots;     /* residual slot pool size */
+    int32_t r_max;       /* largest residual rank a slot holds */
+    int32_t max_tokens;  /* largest batch a segments object accepts */
+    int32_t device;      /* CUDA device ordinal */
+} salt_config;
+
+/*
+ * Residual blob: the unit swapped host -> device (Section "Multi-Tenant
+ * Serving": only the residual is swapped; its size is the paper's "Swap"
+ * column).  A 256-byte header followed by, for each layer l in table order,
+ * At_u[rank][d_in_l] then B_u[rank][d_out_l] (bf16).  payload_bytes =
+ * rank * sum_l (d_in_l + d_out_l) * 2.  layout_hash is FNV-1a 64 over the
+ * (d_in, d_out) pairs as little-endian int32, so a blob built for another
+ * layer table is rejected.
+ */
+typedef struct salt_blob_header {
+    uint64_t magic;          /* SALT_BLOB_MAGIC */
+    uint32_t version;        /* 1 */
+    int32_t rank;            /* 1 .. r_max */
+    int32_t n_layers;
+    float s_u;               /* residual scale */
+    uint64_t payload_bytes;
+    uint64_t layout_hash;
+    uint8_t reserved[SALT_BLOB_HEADER_BYTES - 40];
+} salt_blob_header;
+
+int32_t salt_abi_version(void);
+const char *salt_status_string(salt_status s);
+
+/*
+ * Create a context on config->device: allocates the centroid arena
+ * (n_domains * rc_max * sum(d_in + d_out) bf16), the zeroed residual slot
+ * pool (n_slots slots of header + r_max * sum(d_in + d_out) bf16) and the
+ * device error word.  The context owns all of it until salt_ctx_destroy.
+ * On failure *out is NULL.  Synchronous.
+ */
+salt_status salt_ctx_create(const salt_config *config, salt_ctx **out);
+
+/* Synchronise the device and free everything the context owns.  Segments
+ * objects of the context must be destroyed first.  NULL is a no-op. */
+void salt_ctx_destroy(salt_ctx *ctx);
+
+/* Last error message of the context ("" when none).  Owned by the context. */
+const char *salt_last_error(const salt_ctx *ctx);
+
+/*
+ * Pin domain `domain`'s centroid (Section "Multi-Tenant Serving": the
+ * centroid is loaded once and stays resident).  At_c holds, for each layer
+ * in table order, [rc][d_in_l]; B_c holds, for each layer, [rc][d_out_l]
+ * (bf16).  Either may be host or device memory.  s_c is the centroid scale
+ * (gamma, with any alpha/r folded in).  1 <= rc <= rc_max.  Re-pinning a
+ * domain replaces it.  Synchronous: waits for the device to go idle first,
+ * so no apply in flight reads a half-written centroid.  Setup call, not for
+ * the per-step path.
+ */
+salt_status salt_centroid_pin(salt_ctx *ctx, int32_t domain, int32_t rc,
+                              const void *At_c, const void *B_c, float s_c);
+
+/* Blob size (header + payload) for a rank-`rank` residual over the layer
+ * table of `config`; -1 on an invalid argument.  Host only. */
+int64_t salt_residual_blob_bytes(const salt_config *config, int32_t rank);
+
+/*
+ * Write a blob: header plus At_u (for each layer [rank][d_in_l]) and B_u
+ * (for each layer [rank][d_out_l]), both host arrays of bf16.  blob must
+ * hold salt_residual_blob_bytes(config, rank) bytes (pinned host memory if
+ * it is to be swapped with salt_residual_load).  Host only, synchronous.
+ */
+salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, float s_u,
+                                    const void *At_u, const void *B_u,
+                                    void *blob, int64_t blob_bytes);
+
+/*
+ * Swap a residual into slot `slot` (Section "Multi-Tenant Serving": only
+ * the ultra-low-rank residual moves host -> device).  host_blob must be
+ * page-locked host memory holding a valid blob (checked on the host:
+ * magic, version, rank <= r_max, layer count, layout hash).  Asynchronous
+ * on side_stream: the copy first waits for every apply already enqueued
+ * that reads a segments object referring to `slot`, then one
+ * cudaMemcpyAsync moves the whole blob, then the slot's ready event is
+ * recorded.  The caller keeps host_blob unchanged until side_stream has
+ * passed the copy.  Segments objects built before this call that refer to
+ * `slot` become stale (apply on them returns SALT_ERR_STALE_SEGMENTS until
+ * they are rebuilt).
+ */
+salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob,
+                               salt_stream_t side_stream);
+
+/* Allocate a segments object able to hold max_tokens tokens of this
+ * context (device metadata plus a pinned id staging area).  Synchronous. */
+salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out);
+
+/* Wait for every use of the segments object and free it.  NULL is a no-op. */
+void salt_segments_destroy(salt_segments *seg);
+
+/*
+ * Group a batch (Section "Multi-Tenant Serving": requests are grouped by
+ * their centroid; residuals are batched heterogeneously, as with SGMV in
+ * Section "Multi-Tenant LoRA Serving").  domain_ids and slot_ids are
+ * int32[n_tokens], -1 meaning "no term"; 0 <= n_tokens <= max_tokens.
+ *
+ * If the ids are host memory they are validated here (range, pinned
+ * domain, loaded slot) and errors return at once; the set of slots they
+ * name is recorded so that swaps and applies wait only on what they must.
+ * If they are device memory they are validated by the kernel into the
+ * device error word, and every slot counts as referenced.
+ *
+ * Output (device, owned by seg): tokens stably sorted by (domain, slot),
+ * -1 first, ties in token order; domain runs; user runs; and row blocks
+ * for the apply kernels.  Asynchronous on `stream`; waits for the swaps
+ * of the slots it reads.  Rebuilding a segments object waits for every
+ * apply enqueued on it.
+ */
+salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg,
+                                 const int32_t *domain_ids, const int32_t *slot_ids,
+                                 int32_t n_tokens, salt_stream_t stream);
+
+/*
+ * Copy the segment metadata to host buffers (synchronous; for tests and
+ * diagnostics).  counts[0..3] = n_tokens, domain runs, user runs, row
+ * blocks.  Each array pointer may be NULL; sizes: perm[n_tokens],
+ * dseg_ptr[runs + 1], dseg_dom[runs], useg_ptr[runs + 1], useg_dom[runs],
+ * useg_slot[runs], blocks[3 * blocks] as (start, length, domain) triples.
+ * Buffers of max_tokens + 1 entries (3 * max_tokens for blocks) always
+ * suffice.
+ */
+salt_status salt_segments_export(salt_ctx *ctx, const salt_segments *seg, int32_t *counts,
+                                 int32_t *perm, int32_t *dseg_ptr, int32_t *dseg_dom,
+                                 int32_t *useg_ptr, int32_t *useg_dom, int32_t *useg_slot,
+                                 int32_t *blocks);
+
+/*
+ * Apply centroid + residual LoRA to one layer (Section "Multi-Tenant
+ * Serving", W_final): for every token t of the batch seg was built from,
+ * y[t, :] += s_c (x[t] A_c) B_c + s_u (x[t] a_u) b_u, accumulated in fp32
+ * and rounded once to bf16 (round to nearest even).  x is device
+ * bf16[n_tokens][d_in_layer], y device bf16[n_tokens][d_out_layer], both
+ * 16-byte aligned, rows contiguous; y is read and written in place and
+ * must not overlap x.  Tokens whose ids are both -1 are not touched.
+ * Asynchronous on `stream`.
+ */
+salt_status salt_lora_apply(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
+                            const void *x, void *y, salt_stream_t stream);
+
+/*
+ * The same for n (1..SALT_MAX_GROUP) layers that share the batch, in one
+ * launch: layers[i], x[i], y[i] as in salt_lora_apply.  Use it for
+ * projections that read the same step's activations (q/k/v, gate/up).
+ * The y buffers must not overlap one another or any x.
+ */
+salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int32_t n,
+                                    const int32_t *layers, const void *const *x,
+                                    void *const *y, salt_stream_t stream);
+
+/*
+ * Synchronise `stream`, then read and clear the device error word.
+ * *flags gets the SALT_DEVERR_* bits raised since the last call.  Returns
+ * SALT_ERR_DEVICE_IDS if any bit was set, else SALT_OK.
+ */
+salt_status salt_get_device_error(salt_ctx *ctx, salt_stream_t stream, uint32_t *flags);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SALT_H */

@@ -1,0 +1,646 @@
+// Host runtime behind the C ABI of include/salt.h.
+//
+// Owns the device state of SALT serving (Section "Multi-Tenant Serving"):
+// the centroid arena (pinned once), the fixed residual slot pool filled by
+// host -> device swaps on a side stream, and segments objects.  Ordering
+// between swaps and applies is kept with events only; no call here waits
+// for the device except the setup calls (create, pin, destroy) and the
+// diagnostic ones (export, device error).
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <set>
+#include <string>
+#include <vector>
+
+#include "salt_internal.cuh"
+
+using namespace salt;
+
+struct salt_ctx {
+    int device = 0;
+    int n_layers = 0;
+    std::vector<int32_t> d_in, d_out;
+    std::vector<int64_t> a_off, b_off, res_off;  // elements
+    int64_t sum_din = 0, sum_dout = 0;
+    int n_domains = 0, rc_max = 0, n_slots = 0, r_max = 0, max_tokens = 0;
+    int umax = 1;
+    uint64_t layout_hash = 0;
+
+    uint16_t *arenaA = nullptr, *arenaB = nullptr;
+    int32_t *dom_rc_dev = nullptr;
+    float *dom_sc_dev = nullptr;
+    std::vector<int32_t> dom_rc;
+    std::vector<float> dom_sc;
+
+    uint8_t *pool = nullptr;
+    int64_t slot_stride = 0;
+    std::vector<int32_t> slot_rank;        // 0 = never loaded
+    std::vector<uint64_t> slot_seq;        // loads issued
+    std::vector<cudaEvent_t> slot_ready;
+    std::vector<uint64_t> slot_waited_seq;
+    std::vector<cudaStream_t> slot_waited_stream;
+
+    uint32_t *err_dev = nullptr;
+    int max_active_clusters = 1;
+    std::set<salt_segments *> segs;
+    std::string last_error;
+};
+
+struct salt_segments {
+    salt_ctx *ctx = nullptr;
+    SegDev d{};
+    int32_t *staging[2] = {nullptr, nullptr};  // pinned host [2 * max_tokens]
+    cudaEvent_t staging_ev[2] = {nullptr, nullptr};
+    bool staging_used[2] = {false, false};
+    int staging_next = 0;
+    bool built = false;
+    bool stale = false;
+    bool device_ids = false;
+    int T = 0;
+    int n_blk_max = 0;
+    std::vector<uint8_t> refs;                 // slots named by the last build (host ids)
+    cudaStream_t build_stream = nullptr;
+    std::vector<cudaStream_t> use_streams;     // build stream + apply streams since the build
+    cudaEvent_t built_ev = nullptr;
+    cudaEvent_t tmp_ev = nullptr;
+};
+
+namespace {
+
+salt_status fail(salt_ctx *ctx, salt_status s, const char *fmt, ...)
+{
+    if (ctx) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(buf, sizeof buf, fmt, ap);
+        va_end(ap);
+        ctx->last_error = buf;
+    }
+    return s;
+}
+
+#define CUDA_OR_FAIL(ctx, call)                                                                    \
+    do {                                                                                           \
+        cudaError_t e_ = (call);                                                                   \
+        if (e_ != cudaSuccess)                                                                     \
+            return fail((ctx), SALT_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_));     \
+    } while (0)
+
+uint64_t fnv1a_layout(int n, const int32_t *din, const int32_t *dout)
+{
+    uint64_t h = 1469598103934665603ull;
+    auto mix = [&](int32_t v) {
+        uint32_t u = (uint32_t)v;
+        for (int b = 0; b < 4; ++b) {
+            h ^= (u >> (8 * b)) & 0xffu;
+            h *= 1099511628211ull;
+        }
+    };
+    for (int l = 0; l < n; ++l) {
+        mix(din[l]);
+        mix(dout[l]);
+    }
+    return h;
+}
+
+salt_status check_config(const salt_config *c)
+{
+    if (!c || c->n_layers < 1 || !c->d_in || !c->d_out) return SALT_ERR_INVALID_ARG;
+    for (int l = 0; l < c->n_layers; ++l) {
+        if (c->d_in[l] <= 0 || c->d_out[l] <= 0 || (c->d_in[l] % 8) || (c->d_out[l] % 8))
+            return SALT_ERR_INVALID_ARG;
+    }
+    if (c->n_domains < 0 || c->n_domains >= (1 << 21)) return SALT_ERR_INVALID_ARG;
+    if (c->n_slots < 0 || c->n_slots >= (1 << 21) - 1) return SALT_ERR_INVALID_ARG;
+    if (c->rc_max < 0 || c->rc_max > SALT_MAX_CENTROID_RANK) return SALT_ERR_RANK;
+    if (c->r_max < 1 || c->r_max > SALT_MAX_RESIDUAL_RANK) return SALT_ERR_RANK;
+    if (c->rc_max + c->r_max > S_MAX) return SALT_ERR_RANK;
+    if (c->max_tokens < 1 || c->max_tokens > SALT_MAX_TOKENS) return SALT_ERR_TOO_MANY_TOKENS;
+    return SALT_OK;
+}
+
+int64_t payload_elems(const salt_config *c, int rank)
+{
+    int64_t s = 0;
+    for (int l = 0; l < c->n_layers; ++l) s += (int64_t)c->d_in[l] + c->d_out[l];
+    return s * rank;
+}
+
+bool set_device(salt_ctx *ctx)
+{
+    int cur = -1;
+    if (cudaGetDevice(&cur) != cudaSuccess) return false;
+    if (cur == ctx->device) return true;
+    return cudaSetDevice(ctx->device) == cudaSuccess;
+}
+
+bool is_device_pointer(const void *p)
+{
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+void add_stream(std::vector<cudaStream_t> &v, cudaStream_t s)
+{
+    for (cudaStream_t x : v)
+        if (x == s) return;
+    v.push_back(s);
+}
+
+// Make `stream` wait for all work enqueued so far on the streams that used seg.
+cudaError_t wait_for_uses(salt_segments *seg, cudaStream_t stream)
+{
+    for (cudaStream_t s : seg->use_streams) {
+        if (s == stream) continue;
+        cudaError_t e = cudaEventRecord(seg->tmp_ev, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, seg->tmp_ev, 0);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t salt_abi_version(void) { return SALT_ABI_VERSION; }
+
+const char *salt_status_string(salt_status s)
+{
+    switch (s) {
+    case SALT_OK: return "ok";
+    case SALT_ERR_INVALID_ARG: return "invalid argument";
+    case SALT_ERR_OOM: return "out of memory";
+    case SALT_ERR_NOT_PINNED_HOST: return "host buffer is not page-locked";
+    case SALT_ERR_DOMAIN_NOT_PINNED: return "domain has no pinned centroid";
+    case SALT_ERR_SLOT_RANGE: return "slot id out of range";
+    case SALT_ERR_RANK: return "rank out of range";
+    case SALT_ERR_LAYER_RANGE: return "layer index out of range";
+    case SALT_ERR_ALIGN: return "pointer not 16-byte aligned";
+    case SALT_ERR_BAD_BLOB: return "invalid residual blob";
+    case SALT_ERR_DEVICE_IDS: return "device-side id check failed";
+    case SALT_ERR_TIMEOUT: return "device wait timed out";
+    case SALT_ERR_CUDA: return "CUDA error";
+    case SALT_ERR_SLOT_EMPTY: return "slot was never loaded";
+    case SALT_ERR_TOO_MANY_TOKENS: return "too many tokens";
+    case SALT_ERR_DOMAIN_RANGE: return "domain id out of range";
+    case SALT_ERR_STALE_SEGMENTS: return "segments refer to a slot reloaded after the build";
+    case SALT_ERR_NOT_BUILT: return "segments object not built";
+    }
+    return "unknown status";
+}
+
+const char *salt_last_error(const salt_ctx *ctx) { return ctx ? ctx->last_error.c_str() : "null context"; }
+
+salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
+{
+    if (!out) return SALT_ERR_INVALID_ARG;
+    *out = nullptr;
+    salt_status st = check_config(config);
+    if (st != SALT_OK) return st;
+    salt_ctx *ctx = new (std::nothrow) salt_ctx;
+    if (!ctx) return SALT_ERR_OOM;
+    ctx->device = config->device;
+    if (cudaSetDevice(ctx->device) != cudaSuccess) {
+        cudaGetLastError();
+        delete ctx;
+        return SALT_ERR_CUDA;
+    }
+    ctx->n_layers = config->n_layers;
+    ctx->d_in.assign(config->d_in, config->d_in + config->n_layers);
+    ctx->d_out.assign(config->d_out, config->d_out + config->n_layers);
+    ctx->n_domains = config->n_domains;
+    ctx->rc_max = config->rc_max;
+    ctx->n_slots = config->n_slots;
+    ctx->r_max = config->r_max;
+    ctx->max_tokens = config->max_tokens;
+    ctx->umax = (S_MAX - ctx->rc_max) / ctx->r_max;
+    ctx->layout_hash = fnv1a_layout(ctx->n_layers, config->d_in, config->d_out);
+    int64_t a = 0, b = 0, r = 0;
+    for (int l = 0; l < ctx->n_layers; ++l) {
+        ctx->a_off.push_back(a);
+        ctx->b_off.push_back(b);
+        ctx->res_off.push_back(r);
+        a += (int64_t)ctx->n_domains * ctx->rc_max * ctx->d_in[l];
+        b += (int64_t)ctx->n_domains * ctx->rc_max * ctx->d_out[l];
+        r += (int64_t)ctx->d_in[l] + ctx->d_out[l];
+        ctx->sum_din += ctx->d_in[l];
+        ctx->sum_dout += ctx->d_out[l];
+    }
+    auto cleanup_fail = [&](salt_status s) {
+        salt_ctx_destroy(ctx);
+        return s;
+    };
+    if (a > 0 && cudaMalloc(&ctx->arenaA, (size_t)a * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    if (b > 0 && cudaMalloc(&ctx->arenaB, (size_t)b * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    int nd = ctx->n_domains > 0 ? ctx->n_domains : 1;
+    if (cudaMalloc(&ctx->dom_rc_dev, sizeof(int32_t) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    if (cudaMalloc(&ctx->dom_sc_dev, sizeof(float) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    if (cudaMemset(ctx->dom_rc_dev, 0, sizeof(int32_t) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    if (cudaMemset(ctx->dom_sc_dev, 0, sizeof(float) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    ctx->dom_rc.assign(nd, 0);
+    ctx->dom_sc.assign(nd, 0.f);
+    ctx->slot_stride = (SALT_BLOB_HEADER_BYTES + payload_elems(config, ctx->r_max) * 2 + 255) / 256 * 256;
+    int ns = ctx->n_slots > 0 ? ctx->n_slots : 1;
+    if (cudaMalloc(&ctx->pool, (size_t)ctx->slot_stride * ns) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    if (cudaMemset(ctx->pool, 0, (size_t)ctx->slot_stride * ns) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    ctx->slot_rank.assign(ns, 0);
+    ctx->slot_seq.assign(ns, 0);
+    ctx->slot_waited_seq.assign(ns, 0);
+    ctx->slot_waited_stream.assign(ns, nullptr);
+    ctx->slot_ready.assign(ns, nullptr);
+    for (int s = 0; s < ns; ++s)
+        if (cudaEventCreateWithFlags(&ctx->slot_ready[s], cudaEventDisableTiming) != cudaSuccess)
+            return cleanup_fail(SALT_ERR_CUDA);
+    if (cudaMalloc(&ctx->err_dev, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    if (cudaMemset(ctx->err_dev, 0, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    if (apply_prepare(ctx->device, &ctx->max_active_clusters) != cudaSuccess) {
+        cudaGetLastError();
+        return cleanup_fail(SALT_ERR_CUDA);
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    *out = ctx;
+    return SALT_OK;
+}
+
+void salt_ctx_destroy(salt_ctx *ctx)
+{
+    if (!ctx) return;
+    set_device(ctx);
+    cudaDeviceSynchronize();
+    cudaFree(ctx->arenaA);
+    cudaFree(ctx->arenaB);
+    cudaFree(ctx->dom_rc_dev);
+    cudaFree(ctx->dom_sc_dev);
+    cudaFree(ctx->pool);
+    cudaFree(ctx->err_dev);
+    for (cudaEvent_t e : ctx->slot_ready)
+        if (e) cudaEventDestroy(e);
+    cudaGetLastError();
+    delete ctx;
+}
+
+salt_status salt_centroid_pin(salt_ctx *ctx, int32_t domain, int32_t rc, const void *At_c, const void *B_c,
+                              float s_c)
+{
+    if (!ctx) return SALT_ERR_INVALID_ARG;
+    if (domain < 0 || domain >= ctx->n_domains)
+        return fail(ctx, SALT_ERR_DOMAIN_RANGE, "domain %d outside [0, %d)", domain, ctx->n_domains);
+    if (rc < 1 || rc > ctx->rc_max) return fail(ctx, SALT_ERR_RANK, "centroid rank %d outside [1, %d]", rc, ctx->rc_max);
+    if (!At_c || !B_c) return fail(ctx, SALT_ERR_INVALID_ARG, "null factor pointer");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, cudaDeviceSynchronize());
+    const uint16_t *A = static_cast<const uint16_t *>(At_c);
+    const uint16_t *B = static_cast<const uint16_t *>(B_c);
+    int64_t oa = 0, ob = 0;
+    for (int l = 0; l < ctx->n_layers; ++l) {
+        int64_t na = (int64_t)rc * ctx->d_in[l], nb = (int64_t)rc * ctx->d_out[l];
+        uint16_t *da = ctx->arenaA + ctx->a_off[l] + (int64_t)domain * ctx->rc_max * ctx->d_in[l];
+        uint16_t *db = ctx->arenaB + ctx->b_off[l] + (int64_t)domain * ctx->rc_max * ctx->d_out[l];
+        CUDA_OR_FAIL(ctx, cudaMemcpy(da, A + oa, (size_t)na * 2, cudaMemcpyDefault));
+        CUDA_OR_FAIL(ctx, cudaMemcpy(db, B + ob, (size_t)nb * 2, cudaMemcpyDefault));
+        oa += na;
+        ob += nb;
+    }
+    CUDA_OR_FAIL(ctx, cudaMemcpy(ctx->dom_rc_dev + domain, &rc, sizeof rc, cudaMemcpyHostToDevice));
+    CUDA_OR_FAIL(ctx, cudaMemcpy(ctx->dom_sc_dev + domain, &s_c, sizeof s_c, cudaMemcpyHostToDevice));
+    ctx->dom_rc[domain] = rc;
+    ctx->dom_sc[domain] = s_c;
+    return SALT_OK;
+}
+
+int64_t salt_residual_blob_bytes(const salt_config *config, int32_t rank)
+{
+    if (!config || config->n_layers < 1 || !config->d_in || !config->d_out || rank < 1) return -1;
+    for (int l = 0; l < config->n_layers; ++l)
+        if (config->d_in[l] <= 0 || config->d_out[l] <= 0) return -1;
+    return SALT_BLOB_HEADER_BYTES + payload_elems(config, rank) * 2;
+}
+
+salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, float s_u, const void *At_u,
+                                    const void *B_u, void *blob, int64_t blob_bytes)
+{
+    int64_t need = salt_residual_blob_bytes(config, rank);
+    if (need < 0 || !At_u || !B_u || !blob) return SALT_ERR_INVALID_ARG;
+    if (rank > SALT_MAX_RESIDUAL_RANK) return SALT_ERR_RANK;
+    if (blob_bytes < need) return SALT_ERR_INVALID_ARG;
+    salt_blob_header h;
+    std::memset(&h, 0, sizeof h);
+    h.magic = SALT_BLOB_MAGIC;
+    h.version = 1;
+    h.rank = rank;
+    h.n_layers = config->n_layers;
+    h.s_u = s_u;
+    h.payload_bytes = (uint64_t)payload_elems(config, rank) * 2;
+    h.layout_hash = fnv1a_layout(config->n_layers, config->d_in, config->d_out);
+    uint8_t *out = static_cast<uint8_t *>(blob);
+    std::memcpy(out, &h, sizeof h);
+    uint16_t *pay = reinterpret_cast<uint16_t *>(out + SALT_BLOB_HEADER_BYTES);
+    const uint16_t *A = static_cast<const uint16_t *>(At_u);
+    const uint16_t *B = static_cast<const uint16_t *>(B_u);
+    int64_t oa = 0, ob = 0, op = 0;
+    for (int l = 0; l < config->n_layers; ++l) {
+        int64_t na = (int64_t)rank * config->d_in[l], nb = (int64_t)rank * config->d_out[l];
+        std::memcpy(pay + op, A + oa, (size_t)na * 2);
+        std::memcpy(pay + op + na, B + ob, (size_t)nb * 2);
+        oa += na;
+        ob += nb;
+        op += na + nb;
+    }
+    return SALT_OK;
+}
+
+salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob, salt_stream_t side_stream)
+{
+    if (!ctx) return SALT_ERR_INVALID_ARG;
+    if (slot < 0 || slot >= ctx->n_slots) return fail(ctx, SALT_ERR_SLOT_RANGE, "slot %d outside [0, %d)", slot, ctx->n_slots);
+    if (!host_blob) return fail(ctx, SALT_ERR_INVALID_ARG, "null blob");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, host_blob) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob pointer is not registered with CUDA");
+    }
+    if (attr.type != cudaMemoryTypeHost)
+        return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob is not page-locked host memory (type %d)", (int)attr.type);
+    salt_blob_header h;
+    std::memcpy(&h, host_blob, sizeof h);
+    if (h.magic != SALT_BLOB_MAGIC || h.version != 1) return fail(ctx, SALT_ERR_BAD_BLOB, "bad blob magic or version");
+    if (h.n_layers != ctx->n_layers || h.layout_hash != ctx->layout_hash)
+        return fail(ctx, SALT_ERR_BAD_BLOB, "blob was built for another layer table");
+    if (h.rank < 1 || h.rank > ctx->r_max) return fail(ctx, SALT_ERR_RANK, "blob rank %d outside [1, %d]", h.rank, ctx->r_max);
+    uint64_t pay = (uint64_t)(ctx->sum_din + ctx->sum_dout) * (uint64_t)h.rank * 2;
+    if (h.payload_bytes != pay) return fail(ctx, SALT_ERR_BAD_BLOB, "blob payload size mismatch");
+    cudaStream_t side = static_cast<cudaStream_t>(side_stream);
+
+    // Readers first: every segments object that names this slot waits for its uses.
+    for (salt_segments *seg : ctx->segs) {
+        if (!seg->built) continue;
+        if (!seg->device_ids && !seg->refs[slot]) continue;
+        seg->stale = true;
+        CUDA_OR_FAIL(ctx, wait_for_uses(seg, side));
+    }
+    uint8_t *dst = ctx->pool + (int64_t)slot * ctx->slot_stride;
+    CUDA_OR_FAIL(ctx, cudaMemcpyAsync(dst, host_blob, SALT_BLOB_HEADER_BYTES + pay, cudaMemcpyHostToDevice, side));
+    CUDA_OR_FAIL(ctx, cudaEventRecord(ctx->slot_ready[slot], side));
+    ctx->slot_rank[slot] = h.rank;
+    ctx->slot_seq[slot] += 1;
+    return SALT_OK;
+}
+
+salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
+{
+    if (!ctx || !out) return SALT_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    salt_segments *seg = new (std::nothrow) salt_segments;
+    if (!seg) return SALT_ERR_OOM;
+    seg->ctx = ctx;
+    const int n = ctx->max_tokens;
+    auto alloc = [&](int32_t **p, size_t count) { return cudaMalloc(p, count * sizeof(int32_t)) == cudaSuccess; };
+    bool ok = alloc(&seg->d.ids, 2 * (size_t)n) && alloc(&seg->d.perm, n) && alloc(&seg->d.sorted_slot, n) &&
+              alloc(&seg->d.dseg_ptr, n + 1) && alloc(&seg->d.dseg_dom, n) && alloc(&seg->d.useg_ptr, n + 1) &&
+              alloc(&seg->d.useg_dom, n) && alloc(&seg->d.useg_slot, n) && alloc(&seg->d.blk, 3 * (size_t)n) &&
+              alloc(&seg->d.counts, 4);
+    for (int i = 0; ok && i < 2; ++i) {
+        ok = cudaHostAlloc(&seg->staging[i], 2 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
+             cudaEventCreateWithFlags(&seg->staging_ev[i], cudaEventDisableTiming) == cudaSuccess;
+    }
+    ok = ok && cudaEventCreateWithFlags(&seg->built_ev, cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&seg->tmp_ev, cudaEventDisableTiming) == cudaSuccess;
+    ok = ok && cudaMemset(seg->d.counts, 0, 4 * sizeof(int32_t)) == cudaSuccess;
+    if (!ok) {
+        cudaGetLastError();
+        ctx->segs.insert(seg);
+        salt_segments_destroy(seg);
+        return fail(ctx, SALT_ERR_OOM, "segments allocation failed");
+    }
+    seg->refs.assign(ctx->n_slots > 0 ? ctx->n_slots : 1, 0);
+    ctx->segs.insert(seg);
+    *out = seg;
+    return SALT_OK;
+}
+
+void salt_segments_destroy(salt_segments *seg)
+{
+    if (!seg) return;
+    salt_ctx *ctx = seg->ctx;
+    if (ctx) set_device(ctx);
+    for (cudaStream_t s : seg->use_streams) cudaStreamSynchronize(s);
+    for (int i = 0; i < 2; ++i)
+        if (seg->staging_ev[i]) cudaEventSynchronize(seg->staging_ev[i]);
+    int32_t *arrs[] = {seg->d.ids, seg->d.perm, seg->d.sorted_slot, seg->d.dseg_ptr, seg->d.dseg_dom,
+                       seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_slot, seg->d.blk, seg->d.counts};
+    for (int32_t *p : arrs) cudaFree(p);
+    for (int i = 0; i < 2; ++i) {
+        if (seg->staging[i]) cudaFreeHost(seg->staging[i]);
+        if (seg->staging_ev[i]) cudaEventDestroy(seg->staging_ev[i]);
+    }
+    if (seg->built_ev) cudaEventDestroy(seg->built_ev);
+    if (seg->tmp_ev) cudaEventDestroy(seg->tmp_ev);
+    cudaGetLastError();
+    if (ctx) ctx->segs.erase(seg);
+    delete seg;
+}
+
+salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t *domain_ids,
+                                const int32_t *slot_ids, int32_t n_tokens, salt_stream_t stream_)
+{
+    if (!ctx || !seg || seg->ctx != ctx) return SALT_ERR_INVALID_ARG;
+    if (n_tokens < 0) return fail(ctx, SALT_ERR_INVALID_ARG, "negative token count");
+    if (n_tokens > ctx->max_tokens)
+        return fail(ctx, SALT_ERR_TOO_MANY_TOKENS, "%d tokens > max_tokens %d", n_tokens, ctx->max_tokens);
+    if (n_tokens > 0 && (!domain_ids || !slot_ids)) return fail(ctx, SALT_ERR_INVALID_ARG, "null id array");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    const int T = n_tokens;
+    bool dev_ids = T > 0 && is_device_pointer(domain_ids);
+    if (T > 0 && dev_ids != is_device_pointer(slot_ids))
+        return fail(ctx, SALT_ERR_INVALID_ARG, "domain and slot ids must both be host or both be device memory");
+
+    std::vector<uint8_t> refs;
+    if (!dev_ids) {
+        refs.assign(seg->refs.size(), 0);
+        for (int t = 0; t < T; ++t) {
+            int d = domain_ids[t], s = slot_ids[t];
+            if (d < -1 || d >= ctx->n_domains)
+                return fail(ctx, SALT_ERR_DOMAIN_RANGE, "token %d: domain %d outside [-1, %d)", t, d, ctx->n_domains);
+            if (d >= 0 && ctx->dom_rc[d] == 0)
+                return fail(ctx, SALT_ERR_DOMAIN_NOT_PINNED, "token %d: domain %d has no pinned centroid", t, d);
+            if (s < -1 || s >= ctx->n_slots)
+                return fail(ctx, SALT_ERR_SLOT_RANGE, "token %d: slot %d outside [-1, %d)", t, s, ctx->n_slots);
+            if (s >= 0) {
+                if (ctx->slot_rank[s] == 0)
+                    return fail(ctx, SALT_ERR_SLOT_EMPTY, "token %d: slot %d was never loaded", t, s);
+                refs[s] = 1;
+            }
+        }
+    }
+    // The device buffers of seg may still be read by earlier uses on other streams.
+    CUDA_OR_FAIL(ctx, wait_for_uses(seg, stream));
+    // Swaps of the slots this batch reads must land first.
+    for (int s = 0; s < ctx->n_slots; ++s) {
+        if (!(dev_ids ? true : refs[s])) continue;
+        if (ctx->slot_seq[s] == 0) continue;
+        if (ctx->slot_waited_seq[s] == ctx->slot_seq[s] && ctx->slot_waited_stream[s] == stream) continue;
+        CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(stream, ctx->slot_ready[s], 0));
+        ctx->slot_waited_seq[s] = ctx->slot_seq[s];
+        ctx->slot_waited_stream[s] = stream;
+    }
+    if (T > 0) {
+        if (dev_ids) {
+            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids, domain_ids, (size_t)T * 4, cudaMemcpyDeviceToDevice, stream));
+            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + ctx->max_tokens, slot_ids, (size_t)T * 4,
+                                              cudaMemcpyDeviceToDevice, stream));
+        } else {
+            int k = seg->staging_next;
+            seg->staging_next ^= 1;
+            if (seg->staging_used[k]) CUDA_OR_FAIL(ctx, cudaEventSynchronize(seg->staging_ev[k]));
+            int32_t *h = seg->staging[k];
+            std::memcpy(h, domain_ids, (size_t)T * 4);
+            std::memcpy(h + ctx->max_tokens, slot_ids, (size_t)T * 4);
+            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids, h, (size_t)T * 4, cudaMemcpyHostToDevice, stream));
+            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + ctx->max_tokens, h + ctx->max_tokens, (size_t)T * 4,
+                                              cudaMemcpyHostToDevice, stream));
+            CUDA_OR_FAIL(ctx, cudaEventRecord(seg->staging_ev[k], stream));
+            seg->staging_used[k] = true;
+        }
+    }
+    SegParams p;
+    p.s = seg->d;
+    p.T = T;
+    p.max_tokens = ctx->max_tokens;
+    p.n_domains = ctx->n_domains;
+    p.n_slots = ctx->n_slots;
+    p.r_max = ctx->r_max;
+    p.umax = ctx->umax;
+    p.dom_rc = ctx->dom_rc_dev;
+    p.pool = ctx->pool;
+    p.slot_stride = ctx->slot_stride;
+    p.err = ctx->err_dev;
+    CUDA_OR_FAIL(ctx, launch_segments(p, stream));
+    CUDA_OR_FAIL(ctx, cudaEventRecord(seg->built_ev, stream));
+
+    seg->built = true;
+    seg->stale = false;
+    seg->device_ids = dev_ids;
+    seg->T = T;
+    if (dev_ids) std::fill(seg->refs.begin(), seg->refs.end(), 1);
+    else seg->refs.swap(refs);
+    // row blocks: <= T/TM + groups, groups <= user runs / umax + domain runs (+1 for the skipped run)
+    int64_t bound = (int64_t)T / TM + (int64_t)T / ctx->umax + ctx->n_domains + 3;
+    seg->n_blk_max = (int)(bound < T ? bound : T);
+    seg->build_stream = stream;
+    seg->use_streams.clear();
+    seg->use_streams.push_back(stream);
+    return SALT_OK;
+}
+
+salt_status salt_segments_export(salt_ctx *ctx, const salt_segments *seg, int32_t *counts, int32_t *perm,
+                                 int32_t *dseg_ptr, int32_t *dseg_dom, int32_t *useg_ptr, int32_t *useg_dom,
+                                 int32_t *useg_slot, int32_t *blocks)
+{
+    if (!ctx || !seg || seg->ctx != ctx || !counts) return SALT_ERR_INVALID_ARG;
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, cudaEventSynchronize(seg->built_ev));
+    CUDA_OR_FAIL(ctx, cudaMemcpy(counts, seg->d.counts, 4 * sizeof(int32_t), cudaMemcpyDeviceToHost));
+    const int T = counts[0], nd = counts[1], nu = counts[2], nb = counts[3];
+    auto cp = [&](int32_t *dst, const int32_t *src, int n) -> cudaError_t {
+        if (!dst || n <= 0) return cudaSuccess;
+        return cudaMemcpy(dst, src, (size_t)n * sizeof(int32_t), cudaMemcpyDeviceToHost);
+    };
+    CUDA_OR_FAIL(ctx, cp(perm, seg->d.perm, T));
+    CUDA_OR_FAIL(ctx, cp(dseg_ptr, seg->d.dseg_ptr, nd + 1));
+    CUDA_OR_FAIL(ctx, cp(dseg_dom, seg->d.dseg_dom, nd));
+    CUDA_OR_FAIL(ctx, cp(useg_ptr, seg->d.useg_ptr, nu + 1));
+    CUDA_OR_FAIL(ctx, cp(useg_dom, seg->d.useg_dom, nu));
+    CUDA_OR_FAIL(ctx, cp(useg_slot, seg->d.useg_slot, nu));
+    CUDA_OR_FAIL(ctx, cp(blocks, seg->d.blk, 3 * nb));
+    return SALT_OK;
+}
+
+salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, int32_t n, const int32_t *layers,
+                                    const void *const *x, void *const *y, salt_stream_t stream_)
+{
+    if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
+    salt_segments *seg = const_cast<salt_segments *>(seg_);
+    if (n < 1 || n > SALT_MAX_GROUP || !layers || !x || !y)
+        return fail(ctx, SALT_ERR_INVALID_ARG, "group size %d outside [1, %d] or null arrays", n, SALT_MAX_GROUP);
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (seg->stale) return fail(ctx, SALT_ERR_STALE_SEGMENTS, "a slot named by the segments was reloaded; rebuild");
+    ApplyParams p;
+    std::memset(&p, 0, sizeof p);
+    for (int i = 0; i < n; ++i) {
+        int l = layers[i];
+        if (l < 0 || l >= ctx->n_layers)
+            return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", l, ctx->n_layers);
+        if (seg->T > 0 && (!x[i] || !y[i])) return fail(ctx, SALT_ERR_INVALID_ARG, "null x or y");
+        if ((reinterpret_cast<uintptr_t>(x[i]) | reinterpret_cast<uintptr_t>(y[i])) & 15)
+            return fail(ctx, SALT_ERR_ALIGN, "x / y of group entry %d not 16-byte aligned", i);
+        ApplyProj &pr = p.proj[i];
+        pr.x = static_cast<const uint16_t *>(x[i]);
+        pr.y = static_cast<uint16_t *>(y[i]);
+        pr.A = ctx->arenaA ? ctx->arenaA + ctx->a_off[l] : nullptr;
+        pr.B = ctx->arenaB ? ctx->arenaB + ctx->b_off[l] : nullptr;
+        pr.res_off = ctx->res_off[l];
+        pr.d_in = ctx->d_in[l];
+        pr.d_out = ctx->d_out[l];
+    }
+    if (seg->T == 0) return SALT_OK;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (stream != seg->build_stream) {
+        bool seen = false;
+        for (cudaStream_t s : seg->use_streams) seen |= (s == stream);
+        if (!seen) CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(stream, seg->built_ev, 0));
+    }
+    add_stream(seg->use_streams, stream);
+    p.n_proj = n;
+    p.perm = seg->d.perm;
+    p.sorted_slot = seg->d.sorted_slot;
+    p.blk = seg->d.blk;
+    p.counts = seg->d.counts;
+    p.dom_rc = ctx->dom_rc_dev;
+    p.dom_sc = ctx->dom_sc_dev;
+    p.rc_max = ctx->rc_max;
+    p.pool = ctx->pool;
+    p.slot_stride = ctx->slot_stride;
+    p.r_max = ctx->r_max;
+    p.err = ctx->err_dev;
+    int64_t items = (int64_t)n * seg->n_blk_max;
+    int clusters = (int)(items < ctx->max_active_clusters ? items : ctx->max_active_clusters);
+    if (clusters < 1) clusters = 1;
+    CUDA_OR_FAIL(ctx, launch_apply(p, clusters, stream));
+    return SALT_OK;
+}
+
+salt_status salt_lora_apply(salt_ctx *ctx, const salt_segments *seg, int32_t layer, const void *x, void *y,
+                            salt_stream_t stream)
+{
+    const void *xs[1] = {x};
+    void *ys[1] = {y};
+    return salt_lora_apply_grouped(ctx, seg, 1, &layer, xs, ys, stream);
+}
+
+salt_status salt_get_device_error(salt_ctx *ctx, salt_stream_t stream, uint32_t *flags)
+{
+    if (!ctx || !flags) return SALT_ERR_INVALID_ARG;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    uint32_t v = 0;
+    CUDA_OR_FAIL(ctx, cudaMemcpy(&v, ctx->err_dev, sizeof v, cudaMemcpyDeviceToHost));
+    CUDA_OR_FAIL(ctx, cudaMemset(ctx->err_dev, 0, sizeof v));
+    *flags = v;
+    if (v) return fail(ctx, SALT_ERR_DEVICE_IDS, "device id check raised flags 0x%x", v);
+    return SALT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,268 @@
+// Segment builder: groups a heterogeneous batch for the apply kernel.
+//
+// Section "Multi-Tenant Serving" groups requests by their centroid, and the
+// residuals are batched heterogeneously (SGMV, Section "Multi-Tenant LoRA
+// Serving").  One CTA of 1024 threads:
+//   1. validates every (domain, slot) id into the device error word (an
+//      invalid id is treated as -1, never dereferenced),
+//   2. sorts the keys (domain + 1, slot + 1, token) with a bitonic network in
+//      shared memory; keys are unique, so the order is the stable order of
+//      (domain, slot) with ties in token order and -1 first,
+//   3. writes perm / sorted_slot and the maximal domain and user runs
+//      (two passes over per-thread chunks with a block-wide scan),
+//   4. cuts row blocks for the apply kernel: within a domain run, user runs
+//      are grouped umax at a time and each group is split evenly into
+//      ceil(len / TM) blocks of at most TM tokens.  The leading (-1, -1) run
+//      (tokens with neither term) gets no block, so those rows are never
+//      touched.
+// No global scratch is used: the per-group table lives in the shared memory
+// the keys occupied.
+#include "salt_internal.cuh"
+
+namespace salt {
+namespace {
+
+constexpr int KEY_TOK_BITS = 21;
+constexpr int KEY_SLOT_BITS = 21;
+constexpr uint64_t KEY_TOK_MASK = (1ull << KEY_TOK_BITS) - 1;
+constexpr uint64_t KEY_SLOT_MASK = (1ull << KEY_SLOT_BITS) - 1;
+
+__device__ __forceinline__ int key_dom(uint64_t k) { return (int)(k >> (KEY_TOK_BITS + KEY_SLOT_BITS)) - 1; }
+__device__ __forceinline__ int key_slot(uint64_t k) { return (int)((k >> KEY_TOK_BITS) & KEY_SLOT_MASK) - 1; }
+__device__ __forceinline__ int key_tok(uint64_t k) { return (int)(k & KEY_TOK_MASK); }
+__device__ __forceinline__ uint64_t key_pair(uint64_t k) { return k >> KEY_TOK_BITS; }
+
+// Exclusive scan of one int per thread over the whole block; *total gets the sum.
+__device__ int block_exclusive_scan(int v, int *total, int *warp_sums)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nwarps = blockDim.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < nwarps ? warp_sums[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        warp_sums[lane] = w;  // inclusive
+    }
+    __syncthreads();
+    int before = (warp ? warp_sums[warp - 1] : 0) + x - v;
+    *total = warp_sums[nwarps - 1];
+    __syncthreads();
+    return before;
+}
+
+// Largest index i in [lo, hi) with a[i] <= v (a non-decreasing, a[lo] <= v).
+__device__ __forceinline__ int upper_index(const int32_t *a, int lo, int hi, int v)
+{
+    while (hi - lo > 1) {
+        int mid = (lo + hi) >> 1;
+        if (a[mid] <= v) lo = mid; else hi = mid;
+    }
+    return lo;
+}
+
+__global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
+{
+    extern __shared__ __align__(16) uint64_t keys[];
+    __shared__ int warp_sums[32];
+    const int T = p.T;
+    const int tid = threadIdx.x, nth = blockDim.x;
+
+    if (T == 0) {
+        if (tid == 0) {
+            p.s.dseg_ptr[0] = 0;
+            p.s.useg_ptr[0] = 0;
+            p.s.counts[0] = p.s.counts[1] = p.s.counts[2] = p.s.counts[3] = 0;
+        }
+        return;
+    }
+    int P2 = 1;
+    while (P2 < T) P2 <<= 1;
+
+    // 1. validate and build keys
+    uint32_t errbits = 0;
+    const int32_t *dom_ids = p.s.ids, *slot_ids = p.s.ids + p.max_tokens;
+    for (int i = tid; i < P2; i += nth) {
+        uint64_t key = ~0ull;
+        if (i < T) {
+            int d = dom_ids[i], s = slot_ids[i];
+            if (d < -1 || d >= p.n_domains) {
+                errbits |= SALT_DEVERR_DOMAIN_RANGE;
+                d = -1;
+            } else if (d >= 0 && p.dom_rc[d] <= 0) {
+                errbits |= SALT_DEVERR_DOMAIN_NOT_PINNED;
+                d = -1;
+            }
+            if (s < -1 || s >= p.n_slots) {
+                errbits |= SALT_DEVERR_SLOT_RANGE;
+                s = -1;
+            } else if (s >= 0) {
+                const uint8_t *h = p.pool + (int64_t)s * p.slot_stride;
+                uint64_t magic = *reinterpret_cast<const uint64_t *>(h);
+                int rank = *reinterpret_cast<const int32_t *>(h + 12);
+                if (magic != SALT_BLOB_MAGIC) {
+                    errbits |= SALT_DEVERR_SLOT_EMPTY;
+                    s = -1;
+                } else if (rank < 1 || rank > p.r_max) {
+                    errbits |= SALT_DEVERR_RANK;
+                    s = -1;
+                }
+            }
+            key = ((uint64_t)(d + 1) << (KEY_TOK_BITS + KEY_SLOT_BITS)) |
+                  ((uint64_t)(s + 1) << KEY_TOK_BITS) | (uint64_t)i;
+        }
+        keys[i] = key;
+    }
+    if (errbits) atomicOr(p.err, errbits);
+    __syncthreads();
+
+    // 2. bitonic sort, ascending
+    for (int k = 2; k <= P2; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = tid; i < P2; i += nth) {
+                int ixj = i ^ j;
+                if (ixj > i) {
+                    uint64_t a = keys[i], b = keys[ixj];
+                    bool up = (i & k) == 0;
+                    if ((a > b) == up) {
+                        keys[i] = b;
+                        keys[ixj] = a;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+
+    // 3. runs: count heads per contiguous chunk, scan, then write
+    const int E = (T + nth - 1) / nth;
+    const int lo = min(T, tid * E), hi = min(T, lo + E);
+    int nd = 0, nu = 0;
+    for (int i = lo; i < hi; ++i) {
+        uint64_t k = keys[i];
+        bool dh = i == 0 || key_dom(k) != key_dom(keys[i - 1]);
+        bool uh = i == 0 || key_pair(k) != key_pair(keys[i - 1]);
+        nd += dh;
+        nu += uh;
+    }
+    int n_dseg, n_useg;
+    int od = block_exclusive_scan(nd, &n_dseg, warp_sums);
+    int ou = block_exclusive_scan(nu, &n_useg, warp_sums);
+    for (int i = lo; i < hi; ++i) {
+        uint64_t k = keys[i];
+        int d = key_dom(k), s = key_slot(k);
+        p.s.perm[i] = key_tok(k);
+        p.s.sorted_slot[i] = s;
+        bool dh = i == 0 || d != key_dom(keys[i - 1]);
+        bool uh = i == 0 || key_pair(k) != key_pair(keys[i - 1]);
+        if (dh) {
+            p.s.dseg_ptr[od] = i;
+            p.s.dseg_dom[od] = d;
+            ++od;
+        }
+        if (uh) {
+            p.s.useg_ptr[ou] = i;
+            p.s.useg_dom[ou] = d;
+            p.s.useg_slot[ou] = s;
+            ++ou;
+        }
+    }
+    if (tid == 0) {
+        p.s.dseg_ptr[n_dseg] = T;
+        p.s.useg_ptr[n_useg] = T;
+    }
+    const bool skip0 = key_dom(keys[0]) == -1 && key_slot(keys[0]) == -1;
+    __syncthreads();  // keys are dead from here; run arrays are visible block-wide
+
+    // 4a. group heads over user runs
+    int32_t *grp_first = reinterpret_cast<int32_t *>(keys);  // [n_groups]
+    const int Eu = (n_useg + nth - 1) / nth;
+    const int ulo = min(n_useg, tid * Eu), uhi = min(n_useg, ulo + Eu);
+    auto group_head = [&](int j) -> bool {
+        if (j == 0) return true;
+        if (skip0 && j == 1) return true;
+        int start = p.s.useg_ptr[j];
+        int dr = upper_index(p.s.dseg_ptr, 0, n_dseg, start);
+        int dstart = p.s.dseg_ptr[dr];
+        if (dstart == start) return true;  // first user run of a domain run
+        int first = upper_index(p.s.useg_ptr, 0, n_useg, dstart);
+        int idx = j - first - ((skip0 && dr == 0) ? 1 : 0);
+        return idx % p.umax == 0;
+    };
+    int ng = 0;
+    for (int j = ulo; j < uhi; ++j) ng += group_head(j);
+    int n_groups;
+    int og = block_exclusive_scan(ng, &n_groups, warp_sums);
+    for (int j = ulo; j < uhi; ++j)
+        if (group_head(j)) grp_first[og++] = j;
+    __syncthreads();
+
+    // 4b. blocks per group
+    const int Eg = (n_groups + nth - 1) / nth;
+    const int glo = min(n_groups, tid * Eg), ghi = min(n_groups, glo + Eg);
+    auto group_range = [&](int g, int *start, int *len) {
+        int a = p.s.useg_ptr[grp_first[g]];
+        int b = g + 1 < n_groups ? p.s.useg_ptr[grp_first[g + 1]] : T;
+        *start = a;
+        *len = (g == 0 && skip0) ? 0 : b - a;
+    };
+    int nb = 0;
+    for (int g = glo; g < ghi; ++g) {
+        int a, len;
+        group_range(g, &a, &len);
+        nb += (len + TM - 1) / TM;
+    }
+    int n_blk;
+    int ob = block_exclusive_scan(nb, &n_blk, warp_sums);
+    for (int g = glo; g < ghi; ++g) {
+        int a, len;
+        group_range(g, &a, &len);
+        int q = (len + TM - 1) / TM;
+        int d = p.s.useg_dom[grp_first[g]];
+        for (int b = 0; b < q; ++b) {
+            int s0 = a + (int)(((int64_t)b * len) / q);
+            int s1 = a + (int)(((int64_t)(b + 1) * len) / q);
+            p.s.blk[3 * ob + 0] = s0;
+            p.s.blk[3 * ob + 1] = s1 - s0;
+            p.s.blk[3 * ob + 2] = d;
+            ++ob;
+        }
+    }
+    if (tid == 0) {
+        p.s.counts[0] = T;
+        p.s.counts[1] = n_dseg;
+        p.s.counts[2] = n_useg;
+        p.s.counts[3] = n_blk;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_segments(const SegParams &p, cudaStream_t stream)
+{
+    int P2 = 1;
+    while (P2 < p.T) P2 <<= 1;
+    size_t smem = (size_t)P2 * sizeof(uint64_t);
+    if (smem < 16) smem = 16;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(seg_build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)(SALT_MAX_TOKENS * sizeof(uint64_t)));
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    seg_build_kernel<<<1, SEG_THREADS, smem, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace salt

@@ -1,0 +1,208 @@
+"""ctypes binding of ``libsalt.so`` (the C ABI in ``include/salt.h``).
+
+Argument marshalling only: every function below forwards to the C function
+of the same name; all work runs in the library's CUDA kernels.  Tensors are
+passed by ``data_ptr()``; streams are ``torch.cuda.Stream`` objects (or
+None for the current stream).  A non-OK status raises ``SaltError``.  If
+the library has not been built, importing this module raises ImportError:
+there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libsalt.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with paper_2608_03579_gb300._build.build() "
+                      "(nvcc, sm_103a); there is no CPU fallback")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+STATUS = {
+    0: "SALT_OK", 1: "SALT_ERR_INVALID_ARG", 2: "SALT_ERR_OOM", 3: "SALT_ERR_NOT_PINNED_HOST",
+    4: "SALT_ERR_DOMAIN_NOT_PINNED", 5: "SALT_ERR_SLOT_RANGE", 6: "SALT_ERR_RANK", 7: "SALT_ERR_LAYER_RANGE",
+    8: "SALT_ERR_ALIGN", 9: "SALT_ERR_BAD_BLOB", 10: "SALT_ERR_DEVICE_IDS", 11: "SALT_ERR_TIMEOUT",
+    12: "SALT_ERR_CUDA", 13: "SALT_ERR_SLOT_EMPTY", 14: "SALT_ERR_TOO_MANY_TOKENS", 15: "SALT_ERR_DOMAIN_RANGE",
+    16: "SALT_ERR_STALE_SEGMENTS", 17: "SALT_ERR_NOT_BUILT",
+}
+SALT_BLOB_HEADER_BYTES = 256
+SALT_MAX_TOKENS = 16384
+SALT_MAX_GROUP = 8
+
+
+class SaltError(RuntimeError):
+    def __init__(self, status: int, message: str = ""):
+        self.status = status
+        self.name = STATUS.get(status, f"status {status}")
+        super().__init__(f"{self.name}: {message}" if message else self.name)
+
+
+class salt_config(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("d_in", ctypes.POINTER(ctypes.c_int32)),
+                ("d_out", ctypes.POINTER(ctypes.c_int32)), ("n_domains", ctypes.c_int32),
+                ("rc_max", ctypes.c_int32), ("n_slots", ctypes.c_int32), ("r_max", ctypes.c_int32),
+                ("max_tokens", ctypes.c_int32), ("device", ctypes.c_int32)]
+
+
+_vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+_SIGS = {
+    "salt_abi_version": (_i32, []),
+    "salt_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "salt_ctx_create": (ctypes.c_int, [ctypes.POINTER(salt_config), ctypes.POINTER(_vp)]),
+    "salt_ctx_destroy": (None, [_vp]),
+    "salt_last_error": (ctypes.c_char_p, [_vp]),
+    "salt_centroid_pin": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _f32]),
+    "salt_residual_blob_bytes": (_i64, [ctypes.POINTER(salt_config), _i32]),
+    "salt_residual_blob_pack": (ctypes.c_int, [ctypes.POINTER(salt_config), _i32, _f32, _vp, _vp, _vp, _i64]),
+    "salt_residual_load": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
+    "salt_segments_create": (ctypes.c_int, [_vp, ctypes.POINTER(_vp)]),
+    "salt_segments_destroy": (None, [_vp]),
+    "salt_build_segments": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp]),
+    "salt_segments_export": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "salt_lora_apply": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp]),
+    "salt_lora_apply_grouped": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
+    "salt_get_device_error": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]),
+}
+for _name, (_res, _args) in _SIGS.items():
+    _f = getattr(_lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+def _check(status: int, ctx=None):
+    if status != 0:
+        msg = _lib.salt_last_error(ctx).decode() if ctx else ""
+        raise SaltError(status, msg)
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr(a) -> int | None:
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        assert a.flags.c_contiguous
+        return a.ctypes.data
+    if isinstance(a, int):
+        return a
+    assert a.is_contiguous()
+    return a.data_ptr()
+
+
+def make_config(d_in, d_out, n_domains=0, rc_max=0, n_slots=0, r_max=1, max_tokens=1, device=0):
+    """A salt_config plus the arrays it points to (kept alive on the object)."""
+    din = np.ascontiguousarray(d_in, dtype=np.int32)
+    dout = np.ascontiguousarray(d_out, dtype=np.int32)
+    c = salt_config(len(din), din.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                    dout.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), n_domains, rc_max, n_slots, r_max,
+                    max_tokens, device)
+    c._keep = (din, dout)
+    return c
+
+
+def salt_abi_version() -> int:
+    return int(_lib.salt_abi_version())
+
+
+def salt_status_string(status: int) -> str:
+    return _lib.salt_status_string(status).decode()
+
+
+def salt_ctx_create(d_in, d_out, n_domains, rc_max, n_slots, r_max, max_tokens, device=0) -> int:
+    cfg = make_config(d_in, d_out, n_domains, rc_max, n_slots, r_max, max_tokens, device)
+    out = _vp()
+    _check(_lib.salt_ctx_create(ctypes.byref(cfg), ctypes.byref(out)))
+    return out.value
+
+
+def salt_ctx_destroy(ctx) -> None:
+    _lib.salt_ctx_destroy(ctx)
+
+
+def salt_last_error(ctx) -> str:
+    return _lib.salt_last_error(ctx).decode()
+
+
+def salt_centroid_pin(ctx, domain: int, rc: int, At_c, B_c, s_c: float) -> None:
+    _check(_lib.salt_centroid_pin(ctx, domain, rc, _ptr(At_c), _ptr(B_c), float(s_c)), ctx)
+
+
+def salt_residual_blob_bytes(d_in, d_out, rank: int) -> int:
+    return int(_lib.salt_residual_blob_bytes(ctypes.byref(make_config(d_in, d_out)), rank))
+
+
+def salt_residual_blob_pack(d_in, d_out, rank: int, s_u: float, At_u, B_u, blob, blob_bytes: int) -> None:
+    cfg = make_config(d_in, d_out)
+    _check(_lib.salt_residual_blob_pack(ctypes.byref(cfg), rank, float(s_u), _ptr(At_u), _ptr(B_u),
+                                        _ptr(blob), blob_bytes))
+
+
+def salt_residual_load(ctx, slot: int, host_blob, stream=None) -> None:
+    _check(_lib.salt_residual_load(ctx, slot, _ptr(host_blob), _stream(stream)), ctx)
+
+
+def salt_segments_create(ctx) -> int:
+    out = _vp()
+    _check(_lib.salt_segments_create(ctx, ctypes.byref(out)), ctx)
+    return out.value
+
+
+def salt_segments_destroy(seg) -> None:
+    _lib.salt_segments_destroy(seg)
+
+
+def salt_build_segments(ctx, seg, domain_ids, slot_ids, n_tokens: int | None = None, stream=None) -> None:
+    """ids: numpy / CPU tensors (host path) or CUDA int32 tensors (device path)."""
+    if isinstance(domain_ids, np.ndarray):
+        domain_ids = np.ascontiguousarray(domain_ids, dtype=np.int32)
+        slot_ids = np.ascontiguousarray(slot_ids, dtype=np.int32)
+    n = len(domain_ids) if n_tokens is None else n_tokens
+    _check(_lib.salt_build_segments(ctx, seg, _ptr(domain_ids), _ptr(slot_ids), n, _stream(stream)), ctx)
+
+
+def salt_segments_export(ctx, seg, max_tokens: int) -> dict:
+    n = max_tokens + 1
+    counts = np.zeros(4, dtype=np.int32)
+    arrs = {k: np.zeros(n, dtype=np.int32) for k in
+            ("perm", "dseg_ptr", "dseg_dom", "useg_ptr", "useg_dom", "useg_slot")}
+    blocks = np.zeros(3 * n, dtype=np.int32)
+    _check(_lib.salt_segments_export(ctx, seg, counts.ctypes.data, arrs["perm"].ctypes.data,
+                                     arrs["dseg_ptr"].ctypes.data, arrs["dseg_dom"].ctypes.data,
+                                     arrs["useg_ptr"].ctypes.data, arrs["useg_dom"].ctypes.data,
+                                     arrs["useg_slot"].ctypes.data, blocks.ctypes.data), ctx)
+    T, nd, nu, nb = (int(v) for v in counts)
+    return {"perm": arrs["perm"][:T], "dseg_ptr": arrs["dseg_ptr"][:nd + 1], "dseg_dom": arrs["dseg_dom"][:nd],
+            "useg_ptr": arrs["useg_ptr"][:nu + 1], "useg_dom": arrs["useg_dom"][:nu],
+            "useg_slot": arrs["useg_slot"][:nu], "blocks": blocks[:3 * nb].reshape(nb, 3), "counts": counts}
+
+
+def salt_lora_apply(ctx, seg, layer: int, x, y, stream=None) -> None:
+    _check(_lib.salt_lora_apply(ctx, seg, layer, _ptr(x), _ptr(y), _stream(stream)), ctx)
+
+
+def salt_lora_apply_grouped(ctx, seg, layers, xs, ys, stream=None) -> None:
+    n = len(layers)
+    la = (ctypes.c_int32 * n)(*layers)
+    xa = (ctypes.c_void_p * n)(*[_ptr(t) for t in xs])
+    ya = (ctypes.c_void_p * n)(*[_ptr(t) for t in ys])
+    _check(_lib.salt_lora_apply_grouped(ctx, seg, n, la, xa, ya, _stream(stream)), ctx)
+
+
+def salt_get_device_error(ctx, stream=None, raise_on_flags: bool = False) -> int:
+    flags = ctypes.c_uint32(0)
+    st = _lib.salt_get_device_error(ctx, _stream(stream), ctypes.byref(flags))
+    if st not in (0, 10) or (raise_on_flags and st == 10):
+        _check(st, ctx)
+    return int(flags.value)

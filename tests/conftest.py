@@ -30,3 +30,12 @@ def wl():
     from paper_2608_03579_gb300 import workloads
     workloads.build()
     return workloads
+
+
+@pytest.fixture(scope="session")
+def salt_lib():
+    """Build libsalt.so in-tree (nvcc, sm_103a) and import the binding."""
+    from paper_2608_03579_gb300 import _build
+    _build.build()
+    from paper_2608_03579_gb300 import salt
+    return salt
