@@ -1,0 +1,569 @@
+"""Benchmark of the SALT serving hot path on GB300.
+
+One step = one pass of the whole per-step path over one decode batch of the
+Llama-3.1-8B 32-layer workload (512 tokens, 8 domains with rank-64
+centroids, a 512-slot pool of rank-2 residuals drawn Zipf(1.1)):
+
+  1. 64 new residual blobs are swapped host -> device into the slot region
+     the batch does not read, on a side stream (salt_residual_load),
+  2. the batch is grouped (salt_build_segments, host ids),
+  3. every adapted projection of the 32 layers is applied in place
+     (salt_lora_apply_grouped: q/k/v, o, gate/up, down per layer; 128
+     launches replayed from one CUDA graph).
+
+The swaps overlap the applies (the paper's swap-light serving).  Inputs are
+synthetic, drawn by the seeded generator; nothing comes from a dataset or a
+trained checkpoint.  `value` is tokens/s with x / y resident in HBM; `e2e`
+adds the host <-> device copies of x, y_in and y to every step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--mode salt|rank16]
+
+Under torchrun (N > 1) every rank runs an independent replica on its own
+GPU (the path has no exchange step); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "centroid+residual LoRA apply tokens/s; achieved HBM GB/s as % of GB300 peak"
+WORKLOAD = "llama8b_32layer_decode_step"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="salt", choices=["salt", "reference"])
+    ap.add_argument("--mode", default="salt", choices=["salt", "rank16"])
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ----------------------------------------------------------------------------- distributed
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        torch.cuda.set_device(local)
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+        pg = dist
+    return rank, world, local, pg
+
+
+def barrier(pg, device=None):
+    if pg is not None:
+        import torch
+        if device is not None and pg.get_backend() == "nccl":
+            pg.barrier(device_ids=[device])
+        else:
+            pg.barrier()
+
+
+def max_over_ranks(pg, v: float, device=None) -> float:
+    if pg is None:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64, device=f"cuda:{device}" if pg.get_backend() == "nccl" else "cpu")
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_uuid: str | None, out_path: str | None = None):
+        self.uuid = gpu_uuid
+        self.proc = None
+        self.lines = []
+        self.out_path = out_path
+
+    def __enter__(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+        if self.out_path and self.lines:
+            with open(self.out_path, "w") as f:
+                f.write(self.FIELDS + "\n" + "\n".join(self.lines) + "\n")
+
+    def summary(self):
+        mhz, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                mhz.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+# ----------------------------------------------------------------------------- workload setup
+def groups_of(n_layers):
+    g = []
+    for i in range(n_layers):
+        b = 7 * i
+        g += [[b, b + 1, b + 2], [b + 3], [b + 4, b + 5], [b + 6]]
+    return g
+
+
+class Step:
+    """Device state and per-step actions of the 32-layer decode step."""
+
+    N_ID_SETS = 8
+
+    def __init__(self, args, device: int):
+        import torch
+        from paper_2608_03579_gb300 import workloads as wl
+        from paper_2608_03579_gb300 import salt
+        from paper_2608_03579_gb300.runner import SaltRunner
+
+        self.torch, self.salt, self.wl_mod = torch, salt, wl
+        self.device = device
+        rank16 = args.mode == "rank16"
+        self.rank16 = rank16
+        self.w = wl.config4(seed=4, step=1, n_layers=args.layers, rank16=rank16)
+        self.T = self.w.T
+        self.L = len(self.w.layers)
+        self.groups = groups_of(args.layers)
+        self.ids = [wl.config4_ids(4, s, self.T) for s in range(self.N_ID_SETS)]
+        if rank16:
+            self.ids = [(np.full(self.T, -1, np.int32), sl) for (_, sl) in self.ids]
+        self.runner = SaltRunner(self.w, device=device, max_tokens=self.T)
+        r = self.runner
+        if not rank16:
+            r.pin_centroids()
+        # initial fill of the whole pool; rank-16 mode reuses 64 distinct blobs
+        r_slot = 16 if rank16 else 2
+        nb = r.blob_bytes(r_slot)
+        if rank16:
+            base = [r.make_blob(u, 0, r_slot) for u in range(64)]
+            for u in range(self.w.n_slots):
+                salt.salt_residual_load(r.ctx, u, base[u % 64], None)
+            torch.cuda.synchronize()
+            self.host_sets = [base, base]
+        else:
+            r.load_slots()
+            self.host_sets = [[r.make_blob(wl.config4_region(p) + i, 1 + p) for i in range(wl.C4_REGION)]
+                              for p in range(2)]
+        self.blob_bytes = nb
+        # activations: one contiguous buffer for all projections
+        self.x_off, self.y_off = [], []
+        xo = yo = 0
+        for (_, din, dout) in self.w.layers:
+            self.x_off.append(xo)
+            self.y_off.append(yo)
+            xo += self.T * din
+            yo += self.T * dout
+        self.x_elems, self.y_elems = xo, yo
+        self.x_all = torch.empty(xo, dtype=torch.bfloat16, device=f"cuda:{device}")
+        self.y_all = torch.zeros(yo, dtype=torch.bfloat16, device=f"cuda:{device}")
+        xh = np.empty(xo, dtype=np.uint16)
+        for l in range(self.L):
+            din = self.w.layers[l][1]
+            wl.normal_bf16(self.w.seed, wl.stream_id(wl.K_X, 0, l), self.T * din,
+                           out=xh[self.x_off[l]:self.x_off[l] + self.T * din])
+        self.x_all.copy_(torch.from_numpy(xh.view(np.int16)).view(torch.bfloat16))
+        self.xs = [self.x_all[self.x_off[l]:self.x_off[l] + self.T * self.w.layers[l][1]] for l in range(self.L)]
+        self.ys = [self.y_all[self.y_off[l]:self.y_off[l] + self.T * self.w.layers[l][2]] for l in range(self.L)]
+        self.comp = torch.cuda.Stream(device=device)
+        self.side = torch.cuda.Stream(device=device)
+        self.graph = None
+
+    # one step's actions
+    def swap(self, s):
+        region = self.wl_mod.config4_region(s % self.N_ID_SETS)
+        hs = self.host_sets[s % 2]
+        for i in range(self.wl_mod.C4_REGION):
+            self.salt.salt_residual_load(self.runner.ctx, region + i, hs[i], self.side)
+
+    def build(self, s):
+        dom, slot = self.ids[s % self.N_ID_SETS]
+        self.salt.salt_build_segments(self.runner.ctx, self.runner.seg, dom, slot, stream=self.comp)
+
+    def applies_eager(self, timing=False):
+        torch = self.torch
+        evs = []
+        with torch.cuda.stream(self.comp):
+            for grp in self.groups:
+                if timing:
+                    a = torch.cuda.Event(enable_timing=True)
+                    b = torch.cuda.Event(enable_timing=True)
+                    a.record()
+                self.salt.salt_lora_apply_grouped(self.runner.ctx, self.runner.seg, grp,
+                                                  [self.xs[l] for l in grp], [self.ys[l] for l in grp], self.comp)
+                if timing:
+                    b.record()
+                    evs.append((a, b))
+        return evs
+
+    def capture(self):
+        """One CUDA graph of the 128 grouped applies of a step."""
+        torch = self.torch
+        self.build(0)
+        self.applies_eager()
+        torch.cuda.synchronize(self.device)
+        g = torch.cuda.CUDAGraph()
+        try:
+            with torch.cuda.graph(g, stream=self.comp):
+                for grp in self.groups:
+                    self.salt.salt_lora_apply_grouped(self.runner.ctx, self.runner.seg, grp,
+                                                      [self.xs[l] for l in grp], [self.ys[l] for l in grp],
+                                                      self.comp)
+            self.graph = g
+        except Exception as e:  # graph capture unavailable: eager launches
+            print(f"graph capture failed ({e}); using eager launches", file=sys.stderr)
+            torch.cuda.synchronize(self.device)
+            self.graph = None
+
+    def applies(self):
+        if self.graph is not None:
+            with self.torch.cuda.stream(self.comp):
+                self.graph.replay()
+            return []
+        return self.applies_eager()
+
+    def step(self, s, timing=False):
+        """One whole step; with `timing`, the applies are launched eagerly with a
+        CUDA event pair around each launch (returned)."""
+        self.swap(s)
+        self.build(s)
+        if timing:
+            return self.applies_eager(timing=True)
+        return self.applies()
+
+    def join_side(self):
+        self.comp.wait_stream(self.side)
+
+    def apply_bytes(self):
+        """Algorithmic bytes of one step's applies, per launch group, averaged over the id sets."""
+        per_group = np.zeros(len(self.groups))
+        for dom, slot in self.ids:
+            w = self.w
+            w.dom_ids, w.slot_ids = dom, slot
+            for gi, grp in enumerate(self.groups):
+                per_group[gi] += sum(w.algorithmic_bytes(l) for l in grp)
+        return per_group / len(self.ids)
+
+    def close(self):
+        self.graph = None
+        self.runner.close()
+
+
+# ----------------------------------------------------------------------------- oracle timing
+def oracle_sample(seconds_target: float, mode: str, n_layers: int, tokens: int | None = None):
+    """Time the fp64 oracle on a bounded sample of the same workload: the
+    7 projections of one layer for `tokens` tokens of the batch; scaled to
+    the 32-layer step.  Returns (tokens/s over the full step, sample text, seconds)."""
+    import oracle
+    from paper_2608_03579_gb300 import workloads as wl
+    w = wl.config4(seed=4, step=1, n_layers=1, rank16=(mode == "rank16"))
+    T = w.T
+    n = tokens or T
+    rows = np.arange(n)
+    tables = []
+    for l in range(7):
+        cents = [(w.centroid_At(d, l), w.centroid_B(d, l), 1.0) for d in range(w.n_domains)] if mode != "rank16" else []
+        used = set(int(s) for s in w.slot_ids[rows] if s >= 0)
+        res = [((w.residual_At(u, l), w.residual_B(u, l), 1.0) if u in used else None) for u in range(w.n_slots)]
+        tables.append((w.x(l, rows), w.y_in(l, rows), cents, res))
+    dom = w.dom_ids[rows] if mode != "rank16" else np.full(n, -1, np.int32)
+    t0 = time.perf_counter()
+    for (x, y, cents, res) in tables:
+        oracle.apply(x, y, dom, w.slot_ids[rows], cents, res)
+    dt = time.perf_counter() - t0
+    per_token_step = dt / n * n_layers
+    return 1.0 / per_token_step, f"{n} tokens x the 7 projections of 1 of {n_layers} layers, scaled x{n_layers}", dt
+
+
+# ----------------------------------------------------------------------------- main arms
+def run_reference(args, rank, world, pg):
+    """The oracle arm: the fp64 CPU oracle timed on the host cores."""
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    n_tok = 24
+    for _ in range(args.warmup):
+        oracle_sample(0, args.mode, args.layers, tokens=4)
+    vals, tsum = [], 0.0
+    for _ in range(args.steps):
+        v, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=n_tok)
+        vals.append(v)
+        tsum += dt
+    value = statistics.mean(vals)
+    ms = 1000.0 * 512 / value
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "tokens_per_step": 512, "layers": args.layers,
+                       "projections": 7 * args.layers, "mode": args.mode},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": f"each step: {sample}"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def traffic_from_profile():
+    """Per-launch DRAM traffic from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    p = os.path.join(ROOT, "profiles", "salt_apply_kernel_traffic.json")
+    src = os.path.join(ROOT, "paper_2608_03579_gb300", "csrc", "salt_apply.cu")
+    if not os.path.exists(p):
+        return None, None
+    d = json.load(open(p))
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    if d.get("kernel_source_sha256_16") != h:
+        return None, None
+    return d.get("dram_bytes_per_algorithmic_byte"), d
+
+
+def run_salt(args, rank, world, local, pg):
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(local)
+    peaks, peak_kind = load_peaks()
+    st = Step(args, local)
+    ctx_info = st.salt.salt_ctx_get_info(st.runner.ctx)
+    st.capture()
+    per_group_bytes = st.apply_bytes()
+    step_apply_bytes = float(per_group_bytes.sum())
+    n_launch = len(st.groups)
+
+    # warm-up
+    for s in range(args.warmup):
+        st.step(s)
+    st.join_side()
+    torch.cuda.synchronize(local)
+
+    # timed region: K whole steps
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        if not uuid.startswith("GPU-"):
+            uuid = "GPU-" + uuid
+    except Exception:
+        uuid = None
+    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+    sampler = ClockSampler(uuid, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv"))
+    barrier(pg, local)
+    torch.cuda.synchronize(local)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    with sampler:
+        time.sleep(0.3)
+        t_start.record(st.comp)
+        for s in range(args.warmup, args.warmup + args.steps):
+            st.step(s)
+        st.join_side()
+        t_end.record(st.comp)
+        torch.cuda.synchronize(local)
+        time.sleep(0.2)
+    ms_total = t_start.elapsed_time(t_end)
+    # per-launch durations of the last step (graph-captured event pairs)
+    barrier(pg, local)
+    # per-launch durations of the apply kernel: a pass of whole steps right
+    # after the timed region (swaps still overlapping), with an event pair on
+    # the launching stream around every apply launch
+    n_prof = 3
+    launch_ms = np.zeros(len(st.groups))
+    for s in range(n_prof):
+        evs = st.step(args.warmup + args.steps + s, timing=True)
+        st.join_side()
+        torch.cuda.synchronize(local)
+        launch_ms += np.array([a.elapsed_time(b) for (a, b) in evs])
+    kernel_ms = list(launch_ms / n_prof)
+    kinds = ["qkv", "o", "gate_up", "down"]
+    per_kind = {}
+    for i, k in enumerate(kinds):
+        msk = sum(kernel_ms[i::4])
+        per_kind[k] = {"us_per_launch": 1000.0 * msk / (len(kernel_ms) // 4),
+                       "GB/s": float(per_group_bytes[i::4].sum() / (msk / 1000.0) / 1e9)}
+    # the applies alone (graph replays, no swaps), for context
+    apply_only_ms = None
+    if st.graph is not None:
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(st.comp)
+        for _ in range(5):
+            st.applies()
+        b.record(st.comp)
+        torch.cuda.synchronize(local)
+        apply_only_ms = a.elapsed_time(b) / 5
+    ms_total = max_over_ranks(pg, ms_total, local)
+    ms_per_step = ms_total / args.steps
+    value = world * st.T * args.steps / (ms_total / 1000.0)
+    clocks = sampler.summary()
+
+    # kernel roofline (the apply kernel dominates the step)
+    roof = None
+    if kernel_ms:
+        k_total = sum(kernel_ms)
+        achieved = step_apply_bytes / (k_total / 1000.0) / 1e9
+        ratio, prof = traffic_from_profile()
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"],
+                "traffic": (ratio * step_apply_bytes / n_launch) if ratio else None,
+                "kernel": "salt_apply_kernel", "launches_per_step": n_launch,
+                "algorithmic_bytes_per_launch": step_apply_bytes / n_launch,
+                "avg_launch_us": 1000.0 * k_total / n_launch,
+                "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s"}
+
+    # e2e: host buffers, copies inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        x_host = torch.empty(st.x_elems, dtype=torch.bfloat16, pin_memory=True)
+        x_host.copy_(st.x_all)
+        y_host = torch.zeros(st.y_elems, dtype=torch.bfloat16, pin_memory=True)
+        y_out = torch.empty(st.y_elems, dtype=torch.bfloat16, pin_memory=True)
+        torch.cuda.synchronize(local)
+        n_e2e = max(3, min(args.steps, 10))
+        barrier(pg, local)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(st.comp)
+        for s in range(n_e2e):
+            with torch.cuda.stream(st.comp):
+                st.x_all.copy_(x_host, non_blocking=True)
+                st.y_all.copy_(y_host, non_blocking=True)
+            st.step(args.warmup + args.steps + s)
+            with torch.cuda.stream(st.comp):
+                y_out.copy_(st.y_all, non_blocking=True)
+        st.join_side()
+        e1.record(st.comp)
+        torch.cuda.synchronize(local)
+        e2e_ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / n_e2e
+        h2d = st.x_elems * 2 + st.y_elems * 2 + 2 * st.T * 4 + st.wl_mod.C4_REGION * st.blob_bytes
+        e2e = {"value": world * st.T / (e2e_ms / 1000.0), "unit": "tokens/s", "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(st.y_elems * 2)}
+
+    # swap-only and apply-only reference timings (context for the step time)
+    swap_ms = None
+    try:
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(local)
+        a.record(st.side)
+        for s in range(4):
+            st.swap(args.warmup + s)
+        b.record(st.side)
+        torch.cuda.synchronize(local)
+        swap_ms = a.elapsed_time(b) / 4
+    except Exception:
+        swap_ms = None
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        v1, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=8)
+        n_tok = int(max(8, min(512, 8 * args.cpu_seconds / max(dt, 1e-3))))
+        v, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=n_tok)
+        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": sample + f" ({dt:.1f} s, single-threaded fp64 C)"}
+
+    st.close()
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": WORKLOAD if args.mode == "salt" else WORKLOAD + "_rank16_lora",
+                           "tokens_per_step": st.T, "layers": args.layers, "projections": st.L,
+                           "domains": 8, "centroid_rank": 0 if args.mode == "rank16" else 64,
+                           "residual_rank": 16 if args.mode == "rank16" else 2, "slots": 512,
+                           "swaps_per_step": 64, "swap_bytes_per_step": 64 * st.blob_bytes,
+                           "apply_bytes_per_step": step_apply_bytes,
+                           "l2": "inputs larger than L2 (the step streams > 8 GB; L2 is 126 MB)",
+                           "parallelism": f"replicas x{world}", "launch": "CUDA graph of 128 grouped applies"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": args.steps * (n_launch + 1),
+                "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+                "swap_ms_per_step_alone": swap_ms, "apply_only_ms_per_step": apply_only_ms,
+                "apply_kernel_by_group": per_kind,
+                "apply_launch_shape": {k: ctx_info[k] for k in ("cluster_wide", "cluster_size", "apply_smem_bytes",
+                                                                  "block_tokens", "block_users")}}
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, world, local, pg = dist_setup(args)
+    try:
+        if args.impl == "reference":
+            run_reference(args, rank, world, pg)
+        else:
+            run_salt(args, rank, world, local, pg)
+    finally:
+        if pg is not None:
+            pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -83,6 +83,7 @@ typedef enum salt_status {
 #define SALT_DEVERR_SLOT_RANGE 0x4u
 #define SALT_DEVERR_SLOT_EMPTY 0x8u
 #define SALT_DEVERR_RANK 0x10u
+#define SALT_DEVERR_TIMEOUT 0x20u        /* a bounded in-kernel wait gave up (results of that call invalid) */
 
 /*
  * Context configuration.  d_in / d_out are host arrays of n_layers entries,
@@ -140,6 +141,20 @@ void salt_ctx_destroy(salt_ctx *ctx);
 
 /* Last error message of the context ("" when none).  Owned by the context. */
 const char *salt_last_error(const salt_ctx *ctx);
+
+/* Sizes and launch shape the context chose (diagnostics; no device work). */
+typedef struct salt_ctx_info {
+    int64_t arena_bytes;        /* centroid arena, device */
+    int64_t pool_bytes;         /* residual slot pool, device */
+    int64_t slot_stride;        /* bytes per slot */
+    int32_t cluster_wide;       /* CTAs per shrink cluster when a layer has d_in >= 8192 */
+    int32_t cluster_size;       /* CTAs per shrink cluster otherwise */
+    int32_t apply_smem_bytes;   /* dynamic shared memory per shrink CTA */
+    int32_t block_tokens;       /* max tokens per row block */
+    int32_t block_users;        /* max user runs per row block */
+    int32_t reserved;
+} salt_ctx_info;
+salt_status salt_ctx_get_info(const salt_ctx *ctx, salt_ctx_info *info);
 
 /*
  * Pin domain `domain`'s centroid (Section "Multi-Tenant Serving": the

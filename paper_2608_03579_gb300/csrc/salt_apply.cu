@@ -1,70 +1,81 @@
 // Fused centroid + residual apply (Section "Multi-Tenant Serving":
 // W_final = W_base + gamma * Wbar + delta_i, evaluated in low-rank form).
 //
-// Work unit: one row block (<= TM tokens of one domain, <= umax user runs,
-// from the segment builder) of one projection, handled by a cluster of
-// CLUSTER CTAs.  The block's factors are concatenated into one stack of
+// A row block (<= TM tokens of one domain, <= umax user runs, from the
+// segment builder) concatenates its factors into one stack of
 // S = rc + sum_u r_u rows, [A_c | a_u1 | a_u2 | ...] - the paper's
 // "centroid and residual concatenated into one standard adapter" identity,
-// applied per block - so the whole block is one dense contraction:
+// applied per block - so each block is one dense contraction.  Two kernels:
 //
-//   shrink   V[M x S]   = X[M x d_in] * Stack_A^T     (CTA c: its d_in slice)
-//   reduce   V          = sum over the cluster's partials (DSMEM), then
-//            V_ext[t,s] = s_c V[t,s]         for s < rc
-//                       = s_u(t) V[t,s]      for s in the token's own user's rows
-//                       = 0                  otherwise
-//   expand   Y[M x d_out] += V_ext * Stack_B  (CTA c: its d_out slice)
+//   shrink (one cluster of C CTAs per block and projection; CTA c takes
+//           every C-th 64-wide chunk of d_in):
+//       V^T[S x M] = Stack_A[S x d_in] * X[M x d_in]^T on the tensor cores
+//       (tcgen05.mma, fp32 accumulator in tensor memory; the stack is the
+//       128-row operand, the tokens the N = 16..128 operand), partial sums
+//       reduced across the cluster through distributed shared memory, then
+//       V_ext[t,s] = s_c V[t,s]    for s < rc (centroid rows)
+//                  = s_u V[t,s]    for s in the token's own user's rows
+//                  = 0             otherwise,
+//       rounded to bf16 into the workspace tile of the block.
+//   expand (one CTA per 64 output columns per block, launched as a
+//           programmatic dependent of the shrink):
+//       Y[M x 64] += V_ext * Stack_B[:, cols] (bf16 mma.sync, fp32
+//       accumulation); the B rows and the y rows are fetched before the
+//       dependency wait, so their latency overlaps the shrink.  y is read
+//       once and written once, rounded once (RNE).
 //
-// x rows are gathered by the grouped order, y is read and written once, each
-// factor row is read once per block.  Operands are staged by cp.async in
-// 128-byte-row XOR-swizzled tiles (two stages) and multiplied with bf16
-// mma.sync (fp32 accumulation); V_ext is rounded to bf16 for the expand.
-// The clusters are persistent and stride over (projection, block) items.
-// No global scratch: partial sums live in shared memory.
+// Operands are staged by cp.async in 128-byte-row, 128-byte-swizzled tiles
+// (the layout both ldmatrix and the UMMA descriptors read).  Partial sums
+// never leave the chip; the only scratch is the bf16 V tile per block.
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
 #include "salt_internal.cuh"
+#include "salt_tcgen05.cuh"
 
 namespace cg = cooperative_groups;
 
 namespace salt {
 namespace {
 
-constexpr int KC = 64;                        // K chunk in elements (128-byte rows)
-constexpr int NC = 64;                        // N chunk of the expand
-constexpr int NSTAGE = 2;
-constexpr int TILE_BYTES = TM * 128;          // 128 rows x 128 B
-constexpr int STAGE_BYTES = 2 * TILE_BYTES;   // (X, A) or (Y, B)
-constexpr int STAGES_BYTES = NSTAGE * STAGE_BYTES;
+constexpr int KC = 64;                         // K chunk of the shrink (128-byte rows)
+constexpr int NC = 64;                         // output columns per expand CTA
+constexpr int TILE_BYTES = TM * 128;           // 128 rows x 128 B
+constexpr int STAGES_BYTES = 96 * 1024;        // shrink stage ring
+constexpr int MAX_STAGES = 6;
+constexpr int MAX_CLUSTER = 16;
+constexpr int TMEM_COLS = 128;                 // D^T: up to 128 token columns
 constexpr int PW = SALT_MAX_CENTROID_RANK + SALT_MAX_RESIDUAL_RANK;  // compact partial width
 constexpr int P_BYTES = TM * PW * 4;
-constexpr int RED_ROWS = (TM + CLUSTER - 1) / CLUSTER;
+constexpr int RED_ROWS = TM / CLUSTER;         // rows each CTA reduces (clusters of >= CLUSTER CTAs)
 constexpr int RED_BYTES = RED_ROWS * PW * 4;
-constexpr int VEXT_ROW = S_MAX * 2;           // bytes per V_ext row
-constexpr int VEXT_BYTES = TM * VEXT_ROW;
+constexpr int VT_ROW = VEXT_COLS * 2;          // bytes per V tile row
+constexpr int VT_BYTES = TM * VT_ROW;
 static_assert(P_BYTES + RED_BYTES <= STAGES_BYTES, "partials must fit in the stage area");
-static_assert(S_MAX <= 128 && TM <= 128, "tile shapes");
+static_assert(S_MAX <= 128, "the factor stack is the 128-row UMMA operand");
 
-struct Info {
+struct ShrinkInfo {
     const uint16_t *srcA[S_MAX];  // stacked At rows (element 0 of the row for this layer)
-    const uint16_t *srcB[S_MAX];  // stacked B rows
-    int32_t row[TM];              // x / y row of the i-th token of the block
+    int32_t row[TM];              // x row of the i-th token of the block
     int32_t ucol[TM];             // first stacked row of the token's user, -1: none
     int32_t urank[TM];
     float usu[TM];
-    int32_t wsum[4];
+    int16_t rt0[S_MAX];           // residual stack row -> first token of its user run
+    int16_t rt1[S_MAX];           //                    -> one past the last token
+    int16_t rk[S_MAX];            //                    -> rank index within the user
+    uint64_t bar[MAX_STAGES];     // per stage: the MMAs reading it have completed
+    uint32_t tmem;                // tensor-memory base of D^T
 };
-constexpr int INFO_BYTES = (sizeof(Info) + 127) / 128 * 128;
-constexpr size_t SMEM_BYTES = STAGES_BYTES + VEXT_BYTES + INFO_BYTES;
+struct ExpandInfo {
+    const uint16_t *srcB[S_MAX];  // stacked B rows
+    int32_t row[TM];
+};
+constexpr size_t SHRINK_SMEM = 1024 + STAGES_BYTES + (sizeof(ShrinkInfo) + 127) / 128 * 128;
+constexpr size_t EXPAND_SMEM = 2 * TILE_BYTES + VT_BYTES + (sizeof(ExpandInfo) + 127) / 128 * 128;
 
-__device__ __forceinline__ uint32_t smem_u32(const void *p)
-{
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ int swz128(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
-__device__ __forceinline__ int swz256(int row, int chunk) { return row * VEXT_ROW + ((chunk ^ (row & 7)) << 4); }
+__device__ __forceinline__ int swz256(int row, int chunk) { return row * VT_ROW + ((chunk ^ (row & 7)) << 4); }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid)
 {
@@ -73,7 +84,17 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool v
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+// wait until at most n groups are pending (n in [1, MAX_STAGES - 2])
+__device__ __forceinline__ void cp_async_wait_dyn(int n)
+{
+    switch (n) {
+    case 1: cp_async_wait<1>(); break;
+    case 2: cp_async_wait<2>(); break;
+    case 3: cp_async_wait<3>(); break;
+    default: cp_async_wait<4>(); break;
+    }
+}
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
 {
@@ -93,6 +114,8 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], 
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 
 __device__ __forceinline__ float bf16_to_f(uint16_t h) { return __uint_as_float(((uint32_t)h) << 16); }
 __device__ __forceinline__ uint16_t f_to_bf16(float f)
@@ -101,411 +124,456 @@ __device__ __forceinline__ uint16_t f_to_bf16(float f)
     return *reinterpret_cast<uint16_t *>(&b);
 }
 
-__global__ void __launch_bounds__(APPLY_THREADS, 2) salt_apply_kernel(const __grid_constant__ ApplyParams p)
+// Residual row entry of a block's factor stack -> first element of that row.
+__device__ __forceinline__ const uint16_t *residual_row(const ApplyParams &p, const ApplyProj &pr, int e, bool b_side)
+{
+    const int slot = e >> 8, rank = ((e >> 4) & 15) + 1, k = e & 15;
+    const uint16_t *base = reinterpret_cast<const uint16_t *>(p.pool + (int64_t)slot * p.slot_stride +
+                                                              SALT_BLOB_HEADER_BYTES) + (int64_t)rank * pr.res_off;
+    return b_side ? base + (int64_t)rank * pr.d_in + (int64_t)k * pr.d_out : base + (int64_t)k * pr.d_in;
+}
+
+// ---------------------------------------------------------------------------- shrink
+constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
+
+__global__ void __launch_bounds__(APPLY_THREADS, 2) salt_shrink_kernel(const __grid_constant__ ApplyParams p)
+{
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    // 1024-byte aligned stage ring (the 128-byte swizzle atom of the UMMA operands)
+    uint8_t *stages = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    float *P = reinterpret_cast<float *>(stages);
+    float *RED = reinterpret_cast<float *>(stages + P_BYTES);
+    ShrinkInfo &info = *reinterpret_cast<ShrinkInfo *>(stages + STAGES_BYTES);
+
+    // Before the dependency wait this kernel reads only the segment tables
+    // and the factors: the host launches it as a programmatic dependent only
+    // when the previous kernel on the stream did not write those tables.
+    cg::cluster_group cluster = cg::this_cluster();
+    const int C = (int)cluster.num_blocks();
+    const int crank = (int)cluster.block_rank();
+    const int item = blockIdx.x / C;
+    const int b = item / p.n_proj, pi = item - b * p.n_proj;
+    const int n_blk = p.counts[3];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // every CTA of a cluster takes the same exits, before any cluster barrier
+    if (b >= n_blk || b >= p.blk_cap) {
+        if (b < n_blk && tid == 0 && crank == 0 && pi == 0) atomicOr(p.err, SALT_DEVERR_RANK);
+        pdl_wait();
+        pdl_launch_dependents();
+        return;
+    }
+    const ApplyProj &pr = p.proj[pi];
+    const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
+    const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
+    const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
+    const int S = rc + m1.x;
+    const float s_c = __int_as_float(m1.y);
+    if (S > S_MAX || S == 0) {
+        if (S > S_MAX && tid == 0 && crank == 0) atomicOr(p.err, SALT_DEVERR_RANK);
+        pdl_wait();
+        pdl_launch_dependents();
+        return;
+    }
+    const int d_in = pr.d_in;
+
+    // ---- block setup from the segment tables
+    if (tid < M) {
+        const int t = tid;
+        info.row[t] = p.perm[start + t];
+        const int uo = p.tok_uoff[start + t];
+        const int ur = p.tok_urank[start + t];
+        info.ucol[t] = uo >= 0 ? rc + uo : -1;
+        info.urank[t] = ur;
+        info.usu[t] = p.tok_su[start + t];
+        if (uo >= 0) {
+            const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
+            const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
+            for (int k = 0; k < ur; ++k) {
+                const int s = rc + uo + k;
+                if (s < S_MAX) {
+                    if (head) {
+                        info.rt0[s] = (int16_t)t;
+                        info.rk[s] = (int16_t)k;
+                    }
+                    if (tail) info.rt1[s] = (int16_t)(t + 1);
+                }
+            }
+        }
+    }
+    if (tid < S) {
+        info.srcA[tid] = tid < rc ? pr.A + ((int64_t)d * p.rc_max + tid) * d_in
+                                  : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], false);
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        for (int s = 0; s < MAX_STAGES; ++s) mbar_init(smem_u32(&info.bar[s]), 1);
+        mbar_fence_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = info.tmem;
+
+    // ---- stage geometry: A = the factor stack (always 128 rows: the UMMA M
+    // operand), X = the block's tokens rounded to the 16-row UMMA N step
+    const int m_rows = ((M + 15) >> 4) << 4;
+    const int stage_bytes = TILE_BYTES + m_rows * 128;
+    const int nstage = min(MAX_STAGES, STAGES_BYTES / stage_bytes);
+    const uint32_t ring = smem_u32(stages);
+    const uint32_t idesc = idesc_bf16_f32(128, m_rows);
+
+    // chunks are dealt round-robin over the cluster: at any moment the C CTAs
+    // read adjacent pieces of every row
+    const int nk = (d_in + KC - 1) / KC;
+    const int n_my = nk > crank ? (nk - crank + C - 1) / C : 0;
+
+    // each thread's 16-byte pieces of a chunk, resolved once
+    // piece j of this thread is (row (tid + j*256) / 8, 16-byte chunk tid % 8),
+    // the same for every j, so one column offset serves all pieces
+    const int cb = (tid & 7) * 8;
+    const uint16_t *a_src[MAX_PIECES];
+    const uint16_t *x_src[MAX_PIECES];
+#pragma unroll
+    for (int j = 0; j < MAX_PIECES; ++j) {
+        const int r = (tid + j * APPLY_THREADS) >> 3;
+        a_src[j] = r < S ? info.srcA[r] + cb : nullptr;
+        x_src[j] = r < M ? pr.x + (int64_t)info.row[r] * d_in + cb : nullptr;
+    }
+    auto load_a = [&](int i, int st) {
+        const int k0 = (crank + i * C) * KC;
+        const bool ok = k0 + cb < d_in;
+        const uint32_t base = ring + st * stage_bytes;
+#pragma unroll
+        for (int j = 0; j < MAX_PIECES; ++j) {
+            const int r = (tid + j * APPLY_THREADS) >> 3;
+            if (r < S) cp_async16(base + swz128(r, tid & 7), a_src[j] + (ok ? k0 : 0), ok);
+        }
+    };
+    auto load_x = [&](int i, int st) {
+        const int k0 = (crank + i * C) * KC;
+        const bool ok = k0 + cb < d_in;
+        const uint32_t base = ring + st * stage_bytes + TILE_BYTES;
+#pragma unroll
+        for (int j = 0; j < MAX_PIECES; ++j) {
+            const int r = (tid + j * APPLY_THREADS) >> 3;
+            if (r < M) cp_async16(base + swz128(r, tid & 7), x_src[j] + (ok ? k0 : 0), ok);
+        }
+    };
+
+    // ---- nstage-deep pipeline.  The factor rows of the first chunks are
+    // requested before the dependency wait (no preceding kernel writes them),
+    // x only after it; the first commit group carries those factor rows.
+    bool ok_all = true;
+    for (int s = 0; s < nstage - 1 && s < n_my; ++s) load_a(s, s);
+    pdl_wait();
+    // the expand may start once every CTA has passed the wait: anything it
+    // reads before its own wait (y, B rows) is final by now
+    pdl_launch_dependents();
+    for (int s = 0; s < nstage - 1; ++s) {
+        if (s < n_my) load_x(s, s);
+        cp_async_commit();
+    }
+    for (int it = 0; it < n_my; ++it) {
+        const int st = it % nstage;
+        cp_async_wait_dyn(nstage - 2);
+        fence_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t sa = ring + st * stage_bytes, sx = sa + TILE_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < KC / 16; ++kk)
+                umma_bf16(tmem, sdesc_kmajor_sw128(sa + kk * 32), sdesc_kmajor_sw128(sx + kk * 32), idesc,
+                          (it > 0 || kk > 0) ? 1u : 0u);
+            umma_commit(smem_u32(&info.bar[st]));
+        }
+        const int nxt = it + nstage - 1;
+        if (nxt < n_my) {
+            // the stage of chunk nxt last held chunk it - 1: its MMAs must be done
+            if (it >= 1 && !mbar_wait(smem_u32(&info.bar[(it - 1) % nstage]), ((it - 1) / nstage) & 1))
+                ok_all = false;
+            load_a(nxt, nxt % nstage);
+            load_x(nxt, nxt % nstage);
+        }
+        cp_async_commit();
+    }
+    cp_async_wait<0>();
+    if (n_my > 0 && !mbar_wait(smem_u32(&info.bar[(n_my - 1) % nstage]), ((n_my - 1) / nstage) & 1))
+        ok_all = false;
+    tc_fence_after();
+    __syncthreads();  // the stage ring becomes the partial-sum area
+
+    // ---- D^T (TMEM lanes = stack rows, columns = tokens) -> compact partials:
+    // the centroid rows for every token, a user's rows for that user's tokens
+    if (warp < 4) {
+        const int s = warp * 32 + lane;
+        int col = -1, t0 = 0, t1 = 0;
+        if (s < rc) {
+            col = s;
+            t1 = M;
+        } else if (s < S) {
+            col = rc + info.rk[s];
+            t0 = info.rt0[s];
+            t1 = info.rt1[s];
+        }
+        for (int cg16 = 0; cg16 < (m_rows >> 4); ++cg16) {
+            uint32_t v[16];
+            if (n_my > 0) {
+                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + cg16 * 16, v);
+                tmem_ld_wait();
+            } else {
+#pragma unroll
+                for (int e = 0; e < 16; ++e) v[e] = 0u;
+            }
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = cg16 * 16 + e;
+                if (col >= 0 && t >= t0 && t < t1) P[t * PW + col] = __uint_as_float(v[e]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
+    if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
+    cluster.sync();
+
+    // ---- reduce the rows this CTA owns over the cluster, scale, mask, store V_ext.
+    // All peers' float4 pieces are requested before any is summed; the sum
+    // runs in peer order, so the result does not depend on timing.
+    const int S_pad = (S + 15) & ~15;
+    const int r0 = crank * M / C, r1 = (crank + 1) * M / C;
+    constexpr int PW4 = PW / 4;
+    for (int idx = tid; idx < (r1 - r0) * PW4; idx += APPLY_THREADS) {
+        const int rr = idx / PW4, c4 = idx - rr * PW4, row = r0 + rr;
+        if (c4 * 4 < rc + info.urank[row]) {
+            float4 v[MAX_CLUSTER];
+#pragma unroll
+            for (int qq = 0; qq < MAX_CLUSTER; ++qq)
+                if (qq < C)
+                    v[qq] = *reinterpret_cast<const float4 *>(cluster.map_shared_rank(P, qq) + row * PW + c4 * 4);
+            float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int qq = 0; qq < MAX_CLUSTER; ++qq)
+                if (qq < C) {
+                    s.x += v[qq].x;
+                    s.y += v[qq].y;
+                    s.z += v[qq].z;
+                    s.w += v[qq].w;
+                }
+            *reinterpret_cast<float4 *>(RED + rr * PW + c4 * 4) = s;
+        }
+    }
+    __syncthreads();
+    uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + b) * (TM * VEXT_COLS);
+    const int nch = S_pad >> 3;
+    for (int idx = tid; idx < (r1 - r0) * nch; idx += APPLY_THREADS) {
+        const int rr = idx / nch, c = idx - rr * nch, row = r0 + rr;
+        const int uc = info.ucol[row], ur = info.urank[row];
+        const float us = info.usu[row];
+        uint32_t w[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            uint16_t v2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int col = c * 8 + 2 * h + e;
+                float v = 0.f;
+                if (col < rc) v = s_c * RED[rr * PW + col];
+                else if (uc >= 0 && col >= uc && col < uc + ur) v = us * RED[rr * PW + rc + (col - uc)];
+                v2[e] = f_to_bf16(v);
+            }
+            w[h] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
+        }
+        *reinterpret_cast<uint4 *>(vt + (int64_t)row * VEXT_COLS + c * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    cluster.sync();  // peers have read this CTA's partials
+}
+
+// ---------------------------------------------------------------------------- expand
+__global__ void __launch_bounds__(APPLY_THREADS, 3) salt_expand_kernel(const __grid_constant__ ApplyParams p)
 {
     extern __shared__ __align__(128) uint8_t smem[];
-    uint8_t *stages = smem;
-    float *P = reinterpret_cast<float *>(smem);
-    float *RED = reinterpret_cast<float *>(smem + P_BYTES);
-    uint8_t *vext = smem + STAGES_BYTES;
-    Info &info = *reinterpret_cast<Info *>(smem + STAGES_BYTES + VEXT_BYTES);
+    uint8_t *ys = smem;
+    uint8_t *bs = smem + TILE_BYTES;
+    uint8_t *vs = smem + 2 * TILE_BYTES;
+    ExpandInfo &info = *reinterpret_cast<ExpandInfo *>(smem + 2 * TILE_BYTES + VT_BYTES);
 
-    cg::cluster_group cluster = cg::this_cluster();
-    const int crank = (int)cluster.block_rank();
-    const int cid = blockIdx.x / CLUSTER;
-    const int n_clusters = gridDim.x / CLUSTER;
+    // The next apply's shrink only reads tables and factors before its own
+    // dependency wait, so it may be scheduled as soon as this grid has started.
+    pdl_launch_dependents();
+    const int b = blockIdx.y;
+    const int n_blk = p.counts[3];  // written by the segment kernel, complete before the shrink began
+    if (b >= n_blk || b >= p.blk_cap) return;
+    const int unit = blockIdx.x;
+    int pi = 0;
+    while (pi + 1 < p.n_proj && p.n_unit_prefix[pi + 1] <= unit) ++pi;
+    if (unit >= p.n_unit_prefix[p.n_proj]) return;
+    const ApplyProj &pr = p.proj[pi];
+    const int n0 = (unit - p.n_unit_prefix[pi]) * NC;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g = lane >> 2, q4 = lane & 3;
-    const int n_blk = p.counts[3];
-    const int n_items = n_blk * p.n_proj;
+    const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
+    const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
+    const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
+    const int S = rc + m1.x;
+    if (S > S_MAX || S == 0) return;
+    const int S_pad = (S + 15) & ~15;
+    const int d_out = pr.d_out;
 
-    for (int item = cid; item < n_items; item += n_clusters) {
-        const int pi = item / n_blk, b = item - pi * n_blk;
-        const ApplyProj &pr = p.proj[pi];
-        const int start = p.blk[3 * b], M = p.blk[3 * b + 1], d = p.blk[3 * b + 2];
-        const int rc = d >= 0 ? p.dom_rc[d] : 0;
-        const float s_c = d >= 0 ? p.dom_sc[d] : 0.f;
-        const int d_in = pr.d_in, d_out = pr.d_out;
+    if (tid < M) info.row[tid] = p.perm[start + tid];
+    if (tid < S) {
+        info.srcB[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
+                                  : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], true);
+    }
+    __syncthreads();
 
-        // ---------------- block setup: tokens, users, stacked factor rows
-        int slot = -1, rank = 0, contrib = 0;
-        float su = 0.f;
-        if (tid < M) {
-            info.row[tid] = p.perm[start + tid];
-            int raw = p.sorted_slot[start + tid];
-            if (raw >= 0) {
-                const uint8_t *h = p.pool + (int64_t)raw * p.slot_stride;
-                const salt_blob_header *hd = reinterpret_cast<const salt_blob_header *>(h);
-                if (hd->magic == SALT_BLOB_MAGIC && hd->rank >= 1 && hd->rank <= p.r_max) {
-                    slot = raw;
-                    rank = hd->rank;
-                    su = hd->s_u;
-                } else {
-                    atomicOr(p.err, SALT_DEVERR_SLOT_EMPTY);
+    // independent of the shrink: y rows and stacked B rows of these columns
+    for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
+        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+        bool ok = col < d_out;
+        cp_async16(smem_u32(ys + swz128(r, c)), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
+    }
+    for (int idx = tid; idx < S_pad * 8; idx += APPLY_THREADS) {
+        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+        bool ok = r < S && col < d_out;
+        cp_async16(smem_u32(bs + swz128(r, c)), ok ? info.srcB[r] + col : pr.y, ok);
+    }
+    cp_async_commit();
+
+    // the V tile is produced by the shrink grid
+    pdl_wait();
+    const uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + b) * (TM * VEXT_COLS);
+    const int nch = S_pad >> 3;
+    for (int idx = tid; idx < M * nch; idx += APPLY_THREADS) {
+        int r = idx / nch, c = idx - r * nch;
+        cp_async16(smem_u32(vs + swz256(r, c)), vt + (int64_t)r * VEXT_COLS + c * 8, true);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+
+    const int m_tiles = (M + 15) >> 4;
+    const int em = warp >> 1, en = warp & 1;
+    const int emt0 = em, emt1 = em + 4;
+    const bool eact0 = emt0 < m_tiles, eact1 = emt1 < m_tiles;
+    const uint32_t bs32 = smem_u32(bs), vs32 = smem_u32(vs);
+    float c2[2][4][4];
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) c2[i][j][e] = 0.f;
+    for (int ks = 0; ks < (S_pad >> 4); ++ks) {
+        uint32_t a0[4], a1[4];
+        if (eact0) {
+            int r = emt0 * 16 + (lane & 15);
+            ldsm_x4(vs32 + swz256(r, ks * 2 + (lane >> 4)), a0[0], a0[1], a0[2], a0[3]);
+        }
+        if (eact1) {
+            int r = emt1 * 16 + (lane & 15);
+            ldsm_x4(vs32 + swz256(r, ks * 2 + (lane >> 4)), a1[0], a1[1], a1[2], a1[3]);
+        }
+#pragma unroll
+        for (int np = 0; np < 2; ++np) {
+            const int nt = en * 4 + 2 * np;
+            if (eact0 || eact1) {
+                int mi = lane >> 3;
+                int kr = ks * 16 + (mi & 1) * 8 + (lane & 7);
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(bs32 + swz128(kr, nt + (mi >> 1)), b0, b1, b2, b3);
+                if (eact0) {
+                    mma_bf16(c2[0][2 * np], a0, b0, b1);
+                    mma_bf16(c2[0][2 * np + 1], a0, b2, b3);
                 }
-            }
-            bool head = tid == 0 || raw != p.sorted_slot[start + tid - 1];
-            contrib = (head && slot >= 0) ? rank : 0;
-        }
-        // inclusive scan of contrib over the first TM threads (warps 0..3)
-        int incl = contrib;
-        if (tid < TM) {
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                int y = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += y;
-            }
-            if (lane == 31) info.wsum[warp] = incl;
-        }
-        __syncthreads();
-        int S;
-        {
-            int w0 = info.wsum[0], w1 = info.wsum[1], w2 = info.wsum[2], w3 = info.wsum[3];
-            int before = warp == 0 ? 0 : warp == 1 ? w0 : warp == 2 ? w0 + w1 : w0 + w1 + w2;
-            S = rc + w0 + w1 + w2 + w3;
-            if (tid < M) {
-                int uc = slot >= 0 ? rc + before + incl - rank : -1;
-                info.ucol[tid] = uc;
-                info.urank[tid] = slot >= 0 ? rank : 0;
-                info.usu[tid] = su;
-                if (contrib > 0 && uc + rank <= S_MAX) {
-                    const uint16_t *base = reinterpret_cast<const uint16_t *>(
-                        p.pool + (int64_t)slot * p.slot_stride + SALT_BLOB_HEADER_BYTES) + (int64_t)rank * pr.res_off;
-                    for (int k = 0; k < rank; ++k) {
-                        info.srcA[uc + k] = base + (int64_t)k * d_in;
-                        info.srcB[uc + k] = base + (int64_t)rank * d_in + (int64_t)k * d_out;
-                    }
-                }
-            }
-            if (tid >= TM && tid - TM < rc) {
-                int k = tid - TM;
-                info.srcA[k] = pr.A + ((int64_t)d * p.rc_max + k) * d_in;
-                info.srcB[k] = pr.B + ((int64_t)d * p.rc_max + k) * d_out;
-            }
-        }
-        __syncthreads();
-        // S is computed from the same memory by every CTA of the cluster, so
-        // skipping is uniform and no cluster barrier is left unmatched.
-        if (S > S_MAX || S == 0) {
-            if (S > S_MAX && tid == 0 && crank == 0) atomicOr(p.err, SALT_DEVERR_RANK);
-            __syncthreads();
-            continue;
-        }
-        const int S_pad = (S + 15) & ~15;
-
-        // ---------------- shrink: partial V over this CTA's d_in slice
-        const int nk = (d_in + KC - 1) / KC;
-        const int kc0 = crank * nk / CLUSTER, kc1 = (crank + 1) * nk / CLUSTER;
-        const int m_tiles = (M + 15) >> 4;
-        const int n_nt = S_pad >> 3;
-        const int warps_n = n_nt > 8 ? 2 : 1;
-        const int warps_m = 8 / warps_n;
-        const int wn = warp % warps_n, wm = warp / warps_n;
-        const int nt_lo = wn * 8, nt_hi = min(n_nt, nt_lo + 8);
-        const int mt0 = wm, mt1 = wm + warps_m;
-        const bool act0 = mt0 < m_tiles, act1 = (warps_m == 4) && mt1 < m_tiles;
-
-        float acc[2][8][4];
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) acc[i][j][e] = 0.f;
-
-        auto load_shrink = [&](int kc, int st) {
-            uint8_t *xs = stages + st * STAGE_BYTES;
-            uint8_t *as = xs + TILE_BYTES;
-            const int k0 = kc * KC;
-            for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-                int r = idx >> 3, c = idx & 7, col = k0 + c * 8;
-                bool ok = col < d_in;
-                const uint16_t *src = pr.x + (int64_t)info.row[r] * d_in + (ok ? col : 0);
-                cp_async16(smem_u32(xs + swz128(r, c)), src, ok);
-            }
-            for (int idx = tid; idx < S * 8; idx += APPLY_THREADS) {
-                int r = idx >> 3, c = idx & 7, col = k0 + c * 8;
-                bool ok = col < d_in;
-                cp_async16(smem_u32(as + swz128(r, c)), info.srcA[r] + (ok ? col : 0), ok);
-            }
-        };
-
-        if (kc0 < kc1) {
-            load_shrink(kc0, 0);
-            cp_async_commit();
-            for (int kc = kc0; kc < kc1; ++kc) {
-                const int st = (kc - kc0) & 1;
-                if (kc + 1 < kc1) {
-                    load_shrink(kc + 1, st ^ 1);
-                    cp_async_commit();
-                    cp_async_wait<1>();
-                } else {
-                    cp_async_wait<0>();
-                }
-                __syncthreads();
-                const uint32_t xs = smem_u32(stages + st * STAGE_BYTES);
-                const uint32_t as = xs + TILE_BYTES;
-#pragma unroll
-                for (int kk = 0; kk < KC / 16; ++kk) {
-                    uint32_t a0[4], a1[4];
-                    if (act0) {
-                        int r = mt0 * 16 + (lane & 15);
-                        ldsm_x4(xs + swz128(r, kk * 2 + (lane >> 4)), a0[0], a0[1], a0[2], a0[3]);
-                    }
-                    if (act1) {
-                        int r = mt1 * 16 + (lane & 15);
-                        ldsm_x4(xs + swz128(r, kk * 2 + (lane >> 4)), a1[0], a1[1], a1[2], a1[3]);
-                    }
-#pragma unroll
-                    for (int np = 0; np < 4; ++np) {
-                        const int nt = nt_lo + 2 * np;
-                        if (nt < nt_hi && (act0 || act1)) {
-                            int mi = lane >> 3;
-                            int n = nt * 8 + (mi >> 1) * 8 + (lane & 7);
-                            uint32_t b0, b1, b2, b3;
-                            ldsm_x4(as + swz128(n, kk * 2 + (mi & 1)), b0, b1, b2, b3);
-                            if (act0) {
-                                mma_bf16(acc[0][2 * np], a0, b0, b1);
-                                mma_bf16(acc[0][2 * np + 1], a0, b2, b3);
-                            }
-                            if (act1) {
-                                mma_bf16(acc[1][2 * np], a1, b0, b1);
-                                mma_bf16(acc[1][2 * np + 1], a1, b2, b3);
-                            }
-                        }
-                    }
-                }
-                __syncthreads();
-            }
-        }
-
-        // compact partials: the centroid columns and the token's own user columns
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            const bool act = i == 0 ? act0 : act1;
-            const int mt = i == 0 ? mt0 : mt1;
-            if (!act) continue;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int nt = nt_lo + j;
-                if (nt >= nt_hi) continue;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int row = mt * 16 + g + (e >> 1) * 8;
-                    const int col = nt * 8 + 2 * q4 + (e & 1);
-                    if (row >= M) continue;
-                    if (col < rc) {
-                        P[row * PW + col] = acc[i][j][e];
-                    } else {
-                        const int uc = info.ucol[row];
-                        if (uc >= 0 && col >= uc && col < uc + info.urank[row])
-                            P[row * PW + rc + (col - uc)] = acc[i][j][e];
-                    }
+                if (eact1) {
+                    mma_bf16(c2[1][2 * np], a1, b0, b1);
+                    mma_bf16(c2[1][2 * np + 1], a1, b2, b3);
                 }
             }
         }
-        cluster.sync();
-
-        // ---------------- reduce-scatter over the cluster, then all-gather V_ext
-        const int r0 = crank * M / CLUSTER, r1 = (crank + 1) * M / CLUSTER;
-        for (int idx = tid; idx < (r1 - r0) * PW; idx += APPLY_THREADS) {
-            const int rr = idx / PW, col = idx - rr * PW, row = r0 + rr;
-            if (col < rc + info.urank[row]) {
-                float s = 0.f;
+    }
+    // epilogue: y_in (staged) + delta, one rounding, back into the staged tile
 #pragma unroll
-                for (int qq = 0; qq < CLUSTER; ++qq) {
-                    const float *peer = cluster.map_shared_rank(P, qq);
-                    s += peer[row * PW + col];
-                }
-                RED[rr * PW + col] = s;
+    for (int i = 0; i < 2; ++i) {
+        const bool act = i == 0 ? eact0 : eact1;
+        const int mt = i == 0 ? emt0 : emt1;
+        if (!act) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int nt = en * 4 + j;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int row = mt * 16 + g + h * 8;
+                if (row >= M) continue;
+                uint32_t *cell = reinterpret_cast<uint32_t *>(ys + swz128(row, nt) + q4 * 4);
+                uint32_t v = *cell;
+                float lo = bf16_to_f((uint16_t)(v & 0xffffu)) + c2[i][j][2 * h];
+                float hi = bf16_to_f((uint16_t)(v >> 16)) + c2[i][j][2 * h + 1];
+                *cell = (uint32_t)f_to_bf16(lo) | ((uint32_t)f_to_bf16(hi) << 16);
             }
         }
-        __syncthreads();
-        const int nch = S_pad >> 3;
-        for (int idx = tid; idx < (r1 - r0) * nch; idx += APPLY_THREADS) {
-            const int rr = idx / nch, c = idx - rr * nch, row = r0 + rr;
-            const int uc = info.ucol[row], ur = info.urank[row];
-            const float us = info.usu[row];
-            uint32_t w[4];
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-                uint16_t v2[2];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int col = c * 8 + 2 * h + e;
-                    float v = 0.f;
-                    if (col < rc) v = s_c * RED[rr * PW + col];
-                    else if (uc >= 0 && col >= uc && col < uc + ur) v = us * RED[rr * PW + rc + (col - uc)];
-                    v2[e] = f_to_bf16(v);
-                }
-                w[h] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
-            }
-            const uint4 val = make_uint4(w[0], w[1], w[2], w[3]);
-            const int off = swz256(row, c);
-#pragma unroll
-            for (int qq = 0; qq < CLUSTER; ++qq) {
-                uint8_t *peer = cluster.map_shared_rank(vext, qq);
-                *reinterpret_cast<uint4 *>(peer + off) = val;
-            }
-        }
-        cluster.sync();
-
-        // ---------------- expand: y slice += V_ext * Stack_B
-        const int nn = (d_out + NC - 1) / NC;
-        const int nc0 = crank * nn / CLUSTER, nc1 = (crank + 1) * nn / CLUSTER;
-        const int em = warp >> 1, en = warp & 1;
-        const int emt0 = em, emt1 = em + 4;
-        const bool eact0 = emt0 < m_tiles, eact1 = emt1 < m_tiles;
-
-        auto load_expand = [&](int ncn, int st) {
-            uint8_t *ys = stages + st * STAGE_BYTES;
-            uint8_t *bs = ys + TILE_BYTES;
-            const int n0 = ncn * NC;
-            for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-                int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-                bool ok = col < d_out;
-                const uint16_t *src = pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0);
-                cp_async16(smem_u32(ys + swz128(r, c)), src, ok);
-            }
-            for (int idx = tid; idx < S_pad * 8; idx += APPLY_THREADS) {
-                int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-                bool ok = r < S && col < d_out;
-                const uint16_t *src = ok ? info.srcB[r] + col : pr.y;
-                cp_async16(smem_u32(bs + swz128(r, c)), src, ok);
-            }
-        };
-
-        if (nc0 < nc1) {
-            load_expand(nc0, 0);
-            cp_async_commit();
-            for (int ncn = nc0; ncn < nc1; ++ncn) {
-                const int st = (ncn - nc0) & 1;
-                if (ncn + 1 < nc1) {
-                    load_expand(ncn + 1, st ^ 1);
-                    cp_async_commit();
-                    cp_async_wait<1>();
-                } else {
-                    cp_async_wait<0>();
-                }
-                __syncthreads();
-                uint8_t *ys = stages + st * STAGE_BYTES;
-                const uint32_t ys32 = smem_u32(ys);
-                const uint32_t bs32 = ys32 + TILE_BYTES;
-                const uint32_t vx32 = smem_u32(vext);
-                float c2[2][4][4];
-#pragma unroll
-                for (int i = 0; i < 2; ++i)
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) c2[i][j][e] = 0.f;
-                for (int ks = 0; ks < (S_pad >> 4); ++ks) {
-                    uint32_t a0[4], a1[4];
-                    if (eact0) {
-                        int r = emt0 * 16 + (lane & 15);
-                        ldsm_x4(vx32 + swz256(r, ks * 2 + (lane >> 4)), a0[0], a0[1], a0[2], a0[3]);
-                    }
-                    if (eact1) {
-                        int r = emt1 * 16 + (lane & 15);
-                        ldsm_x4(vx32 + swz256(r, ks * 2 + (lane >> 4)), a1[0], a1[1], a1[2], a1[3]);
-                    }
-#pragma unroll
-                    for (int np = 0; np < 2; ++np) {
-                        const int nt = en * 4 + 2 * np;
-                        if (eact0 || eact1) {
-                            int mi = lane >> 3;
-                            int kr = ks * 16 + (mi & 1) * 8 + (lane & 7);
-                            uint32_t b0, b1, b2, b3;
-                            ldsm_x4_t(bs32 + swz128(kr, nt + (mi >> 1)), b0, b1, b2, b3);
-                            if (eact0) {
-                                mma_bf16(c2[0][2 * np], a0, b0, b1);
-                                mma_bf16(c2[0][2 * np + 1], a0, b2, b3);
-                            }
-                            if (eact1) {
-                                mma_bf16(c2[1][2 * np], a1, b0, b1);
-                                mma_bf16(c2[1][2 * np + 1], a1, b2, b3);
-                            }
-                        }
-                    }
-                }
-                // epilogue: y_in (staged) + delta, one rounding, back into the staged tile
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    const bool act = i == 0 ? eact0 : eact1;
-                    const int mt = i == 0 ? emt0 : emt1;
-                    if (!act) continue;
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const int nt = en * 4 + j;
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const int row = mt * 16 + g + h * 8;
-                            if (row >= M) continue;
-                            uint32_t *cell = reinterpret_cast<uint32_t *>(ys + swz128(row, nt) + q4 * 4);
-                            uint32_t v = *cell;
-                            float lo = bf16_to_f((uint16_t)(v & 0xffffu)) + c2[i][j][2 * h];
-                            float hi = bf16_to_f((uint16_t)(v >> 16)) + c2[i][j][2 * h + 1];
-                            *cell = (uint32_t)f_to_bf16(lo) | ((uint32_t)f_to_bf16(hi) << 16);
-                        }
-                    }
-                }
-                __syncthreads();
-                const int n0 = ncn * NC;
-                for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-                    int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-                    if (col < d_out) {
-                        uint4 v = *reinterpret_cast<const uint4 *>(ys + swz128(r, c));
-                        *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.row[r] * d_out + col) = v;
-                    }
-                }
-                __syncthreads();
-            }
+    }
+    __syncthreads();
+    for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
+        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+        if (col < d_out) {
+            uint4 v = *reinterpret_cast<const uint4 *>(ys + swz128(r, c));
+            *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.row[r] * d_out + col) = v;
         }
     }
 }
 
 }  // namespace
 
-size_t apply_smem_bytes() { return SMEM_BYTES; }
+size_t apply_smem_bytes() { return SHRINK_SMEM; }
 
-cudaError_t apply_prepare(int device, int *max_active_clusters)
+cudaError_t apply_prepare(int device)
 {
     (void)device;
-    cudaError_t e = cudaFuncSetAttribute(salt_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CLUSTER;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(CLUSTER * 64, 1, 1);
-    cfg.blockDim = dim3(APPLY_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = SMEM_BYTES;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    e = cudaOccupancyMaxActiveClusters(&n, salt_apply_kernel, &cfg);
-    if (e != cudaSuccess) return e;
-    *max_active_clusters = n > 0 ? n : 1;
-    return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SHRINK_SMEM);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(salt_expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)EXPAND_SMEM);
+    return e;
 }
 
-cudaError_t launch_apply(const ApplyParams &p, int n_clusters, cudaStream_t stream)
+cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream)
 {
+    if (n_blk_bound <= 0) return cudaSuccess;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CLUSTER;
+    attr[0].val.clusterDim.x = cluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(CLUSTER * n_clusters, 1, 1);
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(cluster * p.n_proj * n_blk_bound, 1, 1);
     cfg.blockDim = dim3(APPLY_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.dynamicSmemBytes = SHRINK_SMEM;
     cfg.stream = stream;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, salt_apply_kernel, p);
+    cfg.numAttrs = shrink_pdl ? 2 : 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, salt_shrink_kernel, p);
+    if (e != cudaSuccess) return e;
+
+    cudaLaunchConfig_t cfg2 = {};
+    cudaLaunchAttribute attr2[1];
+    attr2[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr2[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg2.gridDim = dim3(p.n_unit_prefix[p.n_proj], n_blk_bound, 1);
+    cfg2.blockDim = dim3(APPLY_THREADS, 1, 1);
+    cfg2.dynamicSmemBytes = EXPAND_SMEM;
+    cfg2.stream = stream;
+    cfg2.attrs = attr2;
+    cfg2.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg2, salt_expand_kernel, p);
 }
 
 }  // namespace salt

@@ -15,9 +15,17 @@ namespace salt {
 // rows: rc_max + umax * r_max <= S_MAX.
 constexpr int TM = 128;
 constexpr int S_MAX = 128;
-constexpr int CLUSTER = 8;          // CTAs per row block (split of d_in and d_out)
+constexpr int CLUSTER = 8;          // CTAs per row block in the shrink (split of d_in)
 constexpr int APPLY_THREADS = 256;
 constexpr int SEG_THREADS = 1024;
+
+constexpr int VEXT_COLS = S_MAX;    // row pitch (elements) of a block's V tile in the workspace
+
+// Row-block record (BLK_INTS int32 per block, 32 bytes, read as two int4):
+// first grouped token, token count, domain (-1: none), centroid rank of the
+// domain, residual rows of the factor stack, centroid scale s_c (float bits).
+constexpr int BLK_INTS = 8;
+constexpr int BLK_START = 0, BLK_LEN = 1, BLK_DOM = 2, BLK_RC = 3, BLK_NRES = 4, BLK_SC = 5;
 
 // Device arrays of one segments object.
 struct SegDev {
@@ -29,8 +37,24 @@ struct SegDev {
     int32_t *useg_ptr;     // [max_tokens + 1]
     int32_t *useg_dom;     // [max_tokens]
     int32_t *useg_slot;    // [max_tokens]
-    int32_t *blk;          // [3 * max_tokens] (start, length, domain)
+    int32_t *blk;          // [BLK_INTS * max_tokens], see BLK_* below
     int32_t *counts;       // [4]: n_tokens, domain runs, user runs, row blocks
+    // per grouped token: first stacked row of its user among the block's
+    // residual rows (-1: no residual), the user's rank and scale s_u
+    int32_t *tok_uoff;     // [max_tokens]
+    int32_t *tok_urank;    // [max_tokens]
+    float *tok_su;         // [max_tokens]
+    // per row block: residual rows of the factor stack,
+    // (slot << 8) | ((rank - 1) << 4) | k
+    int32_t *blk_res;      // [max_tokens * S_MAX]
+};
+
+// Scratch of the apply path: one V tile (bf16 [TM][VEXT_COLS]) per
+// (projection of a group, row block), written by the shrink kernel and read
+// by the expand kernel of the same launch pair.
+struct ApplyWork {
+    uint16_t *vext;        // [SALT_MAX_GROUP * blk_cap * TM * VEXT_COLS]
+    int32_t blk_cap;
 };
 
 struct SegParams {
@@ -42,6 +66,7 @@ struct SegParams {
     int32_t r_max;
     int32_t umax;
     const int32_t *dom_rc;   // [n_domains] pinned rank, 0 = not pinned
+    const float *dom_sc;     // [n_domains] centroid scale
     const uint8_t *pool;     // slot pool base
     int64_t slot_stride;     // bytes per slot
     uint32_t *err;           // device error word
@@ -61,23 +86,31 @@ struct ApplyProj {
 struct ApplyParams {
     ApplyProj proj[SALT_MAX_GROUP];
     int32_t n_proj;
+    int32_t n_unit_prefix[SALT_MAX_GROUP + 1];  // expand: 64-column units of projections before p
     const int32_t *perm;
-    const int32_t *sorted_slot;
     const int32_t *blk;
     const int32_t *counts;
-    const int32_t *dom_rc;
-    const float *dom_sc;
+    const int32_t *tok_uoff;
+    const int32_t *tok_urank;
+    const float *tok_su;
+    const int32_t *blk_res;
     int32_t rc_max;
     const uint8_t *pool;
     int64_t slot_stride;
-    int32_t r_max;
+    uint16_t *vext;       // workspace, [n_proj][blk_cap][TM][VEXT_COLS]
+    int32_t blk_cap;
     uint32_t *err;
 };
 
 // Kernel launchers (defined next to the kernels).
 cudaError_t launch_segments(const SegParams &p, cudaStream_t stream);
-cudaError_t apply_prepare(int device, int *max_active_clusters);
-cudaError_t launch_apply(const ApplyParams &p, int n_clusters, cudaStream_t stream);
+cudaError_t apply_prepare(int device);
+// shrink: one cluster of `cluster` CTAs per (row block, projection) for the
+// first n_blk_bound blocks; expand: one CTA per 64 output columns per block,
+// launched as a programmatic dependent of the shrink.  With shrink_pdl the
+// shrink is itself a programmatic dependent of the previous kernel on the
+// stream (only when that kernel did not write the segment tables).
+cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream);
 size_t apply_smem_bytes();
 
 }  // namespace salt

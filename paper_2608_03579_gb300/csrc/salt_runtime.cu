@@ -13,6 +13,7 @@
 #include <set>
 #include <string>
 #include <vector>
+#include <algorithm>
 
 #include "salt_internal.cuh"
 
@@ -43,7 +44,6 @@ struct salt_ctx {
     std::vector<cudaStream_t> slot_waited_stream;
 
     uint32_t *err_dev = nullptr;
-    int max_active_clusters = 1;
     std::set<salt_segments *> segs;
     std::string last_error;
 };
@@ -57,9 +57,11 @@ struct salt_segments {
     int staging_next = 0;
     bool built = false;
     bool stale = false;
+    bool tables_fresh = false;                 // built, and no apply launched since
     bool device_ids = false;
     int T = 0;
-    int n_blk_max = 0;
+    int n_blk_bound = 0;                       // launch bound on the row blocks of the last build
+    ApplyWork work{};                          // V tiles of the apply path
     std::vector<uint8_t> refs;                 // slots named by the last build (host ids)
     cudaStream_t build_stream = nullptr;
     std::vector<cudaStream_t> use_streams;     // build stream + apply streams since the build
@@ -154,6 +156,45 @@ void add_stream(std::vector<cudaStream_t> &v, cudaStream_t s)
     v.push_back(s);
 }
 
+// Row blocks of a T-token batch, whatever the ids: blocks <= T/TM + groups
+// and groups <= user runs / umax + domain runs (+ 1 for the skipped run).
+int block_bound_loose(const salt_ctx *ctx, int T)
+{
+    int64_t b = (int64_t)T / TM + (int64_t)T / ctx->umax + ctx->n_domains + 3;
+    return (int)(b < T ? (b > 0 ? b : 1) : (T > 0 ? T : 1));
+}
+
+// Tighter bound from validated host ids: a domain with n tokens (those
+// with a term) in u user runs yields at most ceil(n / TM) + ceil(u / umax)
+// blocks.  Only sizes the launch grid; the block list itself comes from the
+// segment kernel, and CTAs past its count exit at once.
+int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *slot, int T)
+{
+    std::vector<uint64_t> keys;
+    keys.reserve(T);
+    for (int t = 0; t < T; ++t) {
+        if (dom[t] < 0 && slot[t] < 0) continue;
+        keys.push_back(((uint64_t)(uint32_t)(dom[t] + 1) << 32) | (uint32_t)(slot[t] + 1));
+    }
+    std::sort(keys.begin(), keys.end());
+    int64_t bound = 0;
+    size_t i = 0;
+    while (i < keys.size()) {
+        uint32_t d = (uint32_t)(keys[i] >> 32);
+        int64_t n = 0, u = 0;
+        uint64_t prev = ~0ull;
+        while (i < keys.size() && (uint32_t)(keys[i] >> 32) == d) {
+            if (keys[i] != prev) ++u;
+            prev = keys[i];
+            ++n;
+            ++i;
+        }
+        bound += (n + TM - 1) / TM + (u + ctx->umax - 1) / ctx->umax;
+    }
+    int cap = block_bound_loose(ctx, ctx->max_tokens);
+    return (int)(bound < cap ? bound : cap);
+}
+
 // Make `stream` wait for all work enqueued so far on the streams that used seg.
 cudaError_t wait_for_uses(salt_segments *seg, cudaStream_t stream)
 {
@@ -198,6 +239,21 @@ const char *salt_status_string(salt_status s)
 }
 
 const char *salt_last_error(const salt_ctx *ctx) { return ctx ? ctx->last_error.c_str() : "null context"; }
+
+salt_status salt_ctx_get_info(const salt_ctx *ctx, salt_ctx_info *info)
+{
+    if (!ctx || !info) return SALT_ERR_INVALID_ARG;
+    std::memset(info, 0, sizeof *info);
+    info->arena_bytes = (int64_t)ctx->n_domains * ctx->rc_max * (ctx->sum_din + ctx->sum_dout) * 2;
+    info->pool_bytes = ctx->slot_stride * (int64_t)ctx->n_slots;
+    info->slot_stride = ctx->slot_stride;
+    info->cluster_wide = 16;
+    info->cluster_size = CLUSTER;
+    info->apply_smem_bytes = (int32_t)apply_smem_bytes();
+    info->block_tokens = TM;
+    info->block_users = ctx->umax;
+    return SALT_OK;
+}
 
 salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
 {
@@ -261,7 +317,7 @@ salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
             return cleanup_fail(SALT_ERR_CUDA);
     if (cudaMalloc(&ctx->err_dev, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
     if (cudaMemset(ctx->err_dev, 0, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
-    if (apply_prepare(ctx->device, &ctx->max_active_clusters) != cudaSuccess) {
+    if (apply_prepare(ctx->device) != cudaSuccess) {
         cudaGetLastError();
         return cleanup_fail(SALT_ERR_CUDA);
     }
@@ -407,8 +463,13 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
     auto alloc = [&](int32_t **p, size_t count) { return cudaMalloc(p, count * sizeof(int32_t)) == cudaSuccess; };
     bool ok = alloc(&seg->d.ids, 2 * (size_t)n) && alloc(&seg->d.perm, n) && alloc(&seg->d.sorted_slot, n) &&
               alloc(&seg->d.dseg_ptr, n + 1) && alloc(&seg->d.dseg_dom, n) && alloc(&seg->d.useg_ptr, n + 1) &&
-              alloc(&seg->d.useg_dom, n) && alloc(&seg->d.useg_slot, n) && alloc(&seg->d.blk, 3 * (size_t)n) &&
-              alloc(&seg->d.counts, 4);
+              alloc(&seg->d.useg_dom, n) && alloc(&seg->d.useg_slot, n) &&
+              alloc(&seg->d.blk, (size_t)BLK_INTS * n) && alloc(&seg->d.counts, 4) && alloc(&seg->d.tok_uoff, n) &&
+              alloc(&seg->d.tok_urank, n) && alloc(reinterpret_cast<int32_t **>(&seg->d.tok_su), n) &&
+              alloc(&seg->d.blk_res, (size_t)n * S_MAX);
+    seg->work.blk_cap = block_bound_loose(ctx, n);
+    ok = ok && cudaMalloc(&seg->work.vext, (size_t)SALT_MAX_GROUP * seg->work.blk_cap * TM * VEXT_COLS * 2) ==
+                   cudaSuccess;
     for (int i = 0; ok && i < 2; ++i) {
         ok = cudaHostAlloc(&seg->staging[i], 2 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
              cudaEventCreateWithFlags(&seg->staging_ev[i], cudaEventDisableTiming) == cudaSuccess;
@@ -437,8 +498,11 @@ void salt_segments_destroy(salt_segments *seg)
     for (int i = 0; i < 2; ++i)
         if (seg->staging_ev[i]) cudaEventSynchronize(seg->staging_ev[i]);
     int32_t *arrs[] = {seg->d.ids, seg->d.perm, seg->d.sorted_slot, seg->d.dseg_ptr, seg->d.dseg_dom,
-                       seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_slot, seg->d.blk, seg->d.counts};
+                       seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_slot, seg->d.blk, seg->d.counts,
+                       seg->d.tok_uoff, seg->d.tok_urank, reinterpret_cast<int32_t *>(seg->d.tok_su),
+                       seg->d.blk_res};
     for (int32_t *p : arrs) cudaFree(p);
+    cudaFree(seg->work.vext);
     for (int i = 0; i < 2; ++i) {
         if (seg->staging[i]) cudaFreeHost(seg->staging[i]);
         if (seg->staging_ev[i]) cudaEventDestroy(seg->staging_ev[i]);
@@ -522,6 +586,7 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
     p.r_max = ctx->r_max;
     p.umax = ctx->umax;
     p.dom_rc = ctx->dom_rc_dev;
+    p.dom_sc = ctx->dom_sc_dev;
     p.pool = ctx->pool;
     p.slot_stride = ctx->slot_stride;
     p.err = ctx->err_dev;
@@ -529,14 +594,15 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
     CUDA_OR_FAIL(ctx, cudaEventRecord(seg->built_ev, stream));
 
     seg->built = true;
+    seg->tables_fresh = true;
     seg->stale = false;
     seg->device_ids = dev_ids;
     seg->T = T;
     if (dev_ids) std::fill(seg->refs.begin(), seg->refs.end(), 1);
     else seg->refs.swap(refs);
-    // row blocks: <= T/TM + groups, groups <= user runs / umax + domain runs (+1 for the skipped run)
-    int64_t bound = (int64_t)T / TM + (int64_t)T / ctx->umax + ctx->n_domains + 3;
-    seg->n_blk_max = (int)(bound < T ? bound : T);
+    if (T == 0) seg->n_blk_bound = 0;
+    else if (dev_ids) seg->n_blk_bound = std::min(block_bound_loose(ctx, T), seg->work.blk_cap);
+    else seg->n_blk_bound = std::min(block_bound_host(ctx, domain_ids, slot_ids, T), seg->work.blk_cap);
     seg->build_stream = stream;
     seg->use_streams.clear();
     seg->use_streams.push_back(stream);
@@ -563,7 +629,15 @@ salt_status salt_segments_export(salt_ctx *ctx, const salt_segments *seg, int32_
     CUDA_OR_FAIL(ctx, cp(useg_ptr, seg->d.useg_ptr, nu + 1));
     CUDA_OR_FAIL(ctx, cp(useg_dom, seg->d.useg_dom, nu));
     CUDA_OR_FAIL(ctx, cp(useg_slot, seg->d.useg_slot, nu));
-    CUDA_OR_FAIL(ctx, cp(blocks, seg->d.blk, 3 * nb));
+    if (blocks && nb > 0) {
+        std::vector<int32_t> rec((size_t)BLK_INTS * nb);
+        CUDA_OR_FAIL(ctx, cp(rec.data(), seg->d.blk, BLK_INTS * nb));
+        for (int b = 0; b < nb; ++b) {
+            blocks[3 * b + 0] = rec[(size_t)BLK_INTS * b + BLK_START];
+            blocks[3 * b + 1] = rec[(size_t)BLK_INTS * b + BLK_LEN];
+            blocks[3 * b + 2] = rec[(size_t)BLK_INTS * b + BLK_DOM];
+        }
+    }
     return SALT_OK;
 }
 
@@ -597,28 +671,38 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
     if (seg->T == 0) return SALT_OK;
     if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-    if (stream != seg->build_stream) {
-        bool seen = false;
-        for (cudaStream_t s : seg->use_streams) seen |= (s == stream);
-        if (!seen) CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(stream, seg->built_ev, 0));
-    }
+    // The segments object's V workspace is shared by its applies: applies on
+    // different streams are serialised (no-op for the usual single stream).
+    if (seg->use_streams.size() > 1 || (seg->use_streams.size() == 1 && seg->use_streams[0] != stream))
+        CUDA_OR_FAIL(ctx, wait_for_uses(seg, stream));
     add_stream(seg->use_streams, stream);
     p.n_proj = n;
+    int units = 0, max_din = 0;
+    for (int i = 0; i < n; ++i) {
+        p.n_unit_prefix[i] = units;
+        units += (p.proj[i].d_out + 63) / 64;
+        max_din = std::max(max_din, p.proj[i].d_in);
+    }
+    p.n_unit_prefix[n] = units;
     p.perm = seg->d.perm;
-    p.sorted_slot = seg->d.sorted_slot;
     p.blk = seg->d.blk;
     p.counts = seg->d.counts;
-    p.dom_rc = ctx->dom_rc_dev;
-    p.dom_sc = ctx->dom_sc_dev;
+    p.tok_uoff = seg->d.tok_uoff;
+    p.tok_urank = seg->d.tok_urank;
+    p.tok_su = seg->d.tok_su;
+    p.blk_res = seg->d.blk_res;
     p.rc_max = ctx->rc_max;
     p.pool = ctx->pool;
     p.slot_stride = ctx->slot_stride;
-    p.r_max = ctx->r_max;
+    p.vext = seg->work.vext;
+    p.blk_cap = seg->work.blk_cap;
     p.err = ctx->err_dev;
-    int64_t items = (int64_t)n * seg->n_blk_max;
-    int clusters = (int)(items < ctx->max_active_clusters ? items : ctx->max_active_clusters);
-    if (clusters < 1) clusters = 1;
-    CUDA_OR_FAIL(ctx, launch_apply(p, clusters, stream));
+    // wide inputs split d_in over 16 CTAs so each streams a shorter slice
+    const int cluster = max_din >= 8192 ? 16 : CLUSTER;
+    // The first apply after a build waits for the segment kernel in full;
+    // later ones overlap their table reads with the previous kernel.
+    CUDA_OR_FAIL(ctx, launch_apply(p, seg->n_blk_bound, cluster, !seg->tables_fresh, stream));
+    seg->tables_fresh = false;
     return SALT_OK;
 }
 

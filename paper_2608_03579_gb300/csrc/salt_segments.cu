@@ -232,9 +232,12 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         for (int b = 0; b < q; ++b) {
             int s0 = a + (int)(((int64_t)b * len) / q);
             int s1 = a + (int)(((int64_t)(b + 1) * len) / q);
-            p.s.blk[3 * ob + 0] = s0;
-            p.s.blk[3 * ob + 1] = s1 - s0;
-            p.s.blk[3 * ob + 2] = d;
+            int32_t *rec = p.s.blk + (int64_t)BLK_INTS * ob;
+            rec[BLK_START] = s0;
+            rec[BLK_LEN] = s1 - s0;
+            rec[BLK_DOM] = d;
+            rec[BLK_RC] = d >= 0 ? p.dom_rc[d] : 0;
+            rec[BLK_SC] = __float_as_int(d >= 0 ? p.dom_sc[d] : 0.f);
             ++ob;
         }
     }
@@ -243,6 +246,51 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         p.s.counts[1] = n_dseg;
         p.s.counts[2] = n_useg;
         p.s.counts[3] = n_blk;
+    }
+    __syncthreads();
+
+    // 5. per-block factor stacks: the residual rows of block b are the rows
+    //    of its user runs in order, (slot << 8) | ((rank - 1) << 4) | k; each
+    //    token records where its own user's rows start.  One warp per block.
+    const int lane = tid & 31, warp = tid >> 5, nwarp = nth >> 5;
+    for (int b = warp; b < n_blk; b += nwarp) {
+        const int s0 = p.s.blk[BLK_INTS * b + BLK_START], M = p.s.blk[BLK_INTS * b + BLK_LEN];
+        int carry = 0;
+        for (int base = 0; base < M; base += 32) {
+            const int i = base + lane;
+            int slot = -1, rank = 0, contrib = 0;
+            float su = 0.f;
+            if (i < M) {
+                slot = p.s.sorted_slot[s0 + i];
+                if (slot >= 0) {
+                    const salt_blob_header *h =
+                        reinterpret_cast<const salt_blob_header *>(p.pool + (int64_t)slot * p.slot_stride);
+                    rank = h->rank;
+                    su = h->s_u;
+                }
+                bool head = i == 0 || slot != p.s.sorted_slot[s0 + i - 1];
+                contrib = (head && slot >= 0) ? rank : 0;
+            }
+            int incl = contrib;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                int y = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const int total = __shfl_sync(0xffffffffu, incl, 31);
+            if (i < M) {
+                const int off = carry + incl - rank;
+                p.s.tok_uoff[s0 + i] = slot >= 0 ? off : -1;
+                p.s.tok_urank[s0 + i] = rank;
+                p.s.tok_su[s0 + i] = su;
+                if (contrib > 0)
+                    for (int k = 0; k < rank; ++k)
+                        if (off + k < S_MAX)
+                            p.s.blk_res[(int64_t)b * S_MAX + off + k] = (slot << 8) | ((rank - 1) << 4) | k;
+            }
+            carry += total;
+        }
+        if (lane == 0) p.s.blk[BLK_INTS * b + BLK_NRES] = carry;
     }
 }
 
@@ -254,12 +302,17 @@ cudaError_t launch_segments(const SegParams &p, cudaStream_t stream)
     while (P2 < p.T) P2 <<= 1;
     size_t smem = (size_t)P2 * sizeof(uint64_t);
     if (smem < 16) smem = 16;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(seg_build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)(SALT_MAX_TOKENS * sizeof(uint64_t)));
+    // the attribute is per device; set it once for each device used
+    static unsigned long long configured = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(configured & bit)) {
+        e = cudaFuncSetAttribute(seg_build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(SALT_MAX_TOKENS * sizeof(uint64_t)));
         if (e != cudaSuccess) return e;
-        configured = true;
+        configured |= bit;
     }
     seg_build_kernel<<<1, SEG_THREADS, smem, stream>>>(p);
     return cudaGetLastError();

@@ -49,6 +49,13 @@ class salt_config(ctypes.Structure):
                 ("max_tokens", ctypes.c_int32), ("device", ctypes.c_int32)]
 
 
+class salt_ctx_info(ctypes.Structure):
+    _fields_ = [("arena_bytes", ctypes.c_int64), ("pool_bytes", ctypes.c_int64), ("slot_stride", ctypes.c_int64),
+                ("cluster_wide", ctypes.c_int32), ("cluster_size", ctypes.c_int32),
+                ("apply_smem_bytes", ctypes.c_int32), ("block_tokens", ctypes.c_int32),
+                ("block_users", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
 _SIGS = {
     "salt_abi_version": (_i32, []),
@@ -56,6 +63,7 @@ _SIGS = {
     "salt_ctx_create": (ctypes.c_int, [ctypes.POINTER(salt_config), ctypes.POINTER(_vp)]),
     "salt_ctx_destroy": (None, [_vp]),
     "salt_last_error": (ctypes.c_char_p, [_vp]),
+    "salt_ctx_get_info": (ctypes.c_int, [_vp, ctypes.POINTER(salt_ctx_info)]),
     "salt_centroid_pin": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _f32]),
     "salt_residual_blob_bytes": (_i64, [ctypes.POINTER(salt_config), _i32]),
     "salt_residual_blob_pack": (ctypes.c_int, [ctypes.POINTER(salt_config), _i32, _f32, _vp, _vp, _vp, _i64]),
@@ -133,6 +141,12 @@ def salt_ctx_destroy(ctx) -> None:
 
 def salt_last_error(ctx) -> str:
     return _lib.salt_last_error(ctx).decode()
+
+
+def salt_ctx_get_info(ctx) -> dict:
+    info = salt_ctx_info()
+    _check(_lib.salt_ctx_get_info(ctx, ctypes.byref(info)), ctx)
+    return {k: getattr(info, k) for (k, _) in salt_ctx_info._fields_ if k != "reserved"}
 
 
 def salt_centroid_pin(ctx, domain: int, rc: int, At_c, B_c, s_c: float) -> None:
