@@ -266,6 +266,30 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
                                     void *const *y, salt_stream_t stream);
 
 /*
+ * salt_lora_apply for callers that cannot allocate device memory when they
+ * apply - for example a serving engine whose device memory is planned up
+ * front and that forbids allocations once serving starts, or code that
+ * runs where cudaMalloc is not allowed.  (The paper has no counterpart;
+ * this is a deployment convenience of the library.)
+ *
+ * Same arguments, result and ordering as salt_lora_apply, for one layer.
+ * The intermediate V tiles live in a static device array of this library
+ * (2 MiB, held by every device that loads the library until the process
+ * exits) instead of the segments object's workspace; the call itself
+ * allocates nothing.  Limit: the batch may need at most 64 row blocks
+ * (blocks hold <= 128 tokens of one domain); a larger batch returns
+ * SALT_ERR_TOO_MANY_TOKENS before any device work.  The first call on a
+ * device looks up the array's device address (cudaGetSymbolAddress); make
+ * that first call before any stream capture.  Every call shares the one
+ * array: calls that may overlap on the GPU (on different streams, or from
+ * different contexts or threads) race on it and must be serialised by the
+ * caller.  Nothing in the array needs to start at zero: each call writes
+ * every entry it later reads.
+ */
+salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
+                                   const void *x, void *y, salt_stream_t stream);
+
+/*
  * Synchronise `stream`, then read and clear the device error word.
  * *flags gets the SALT_DEVERR_* bits raised since the last call.  Returns
  * SALT_ERR_DEVICE_IDS if any bit was set, else SALT_OK.

@@ -30,6 +30,8 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
 
@@ -528,9 +530,35 @@ __global__ void __launch_bounds__(APPLY_THREADS, 3) salt_expand_kernel(const __g
     }
 }
 
+// Scratch of salt_lora_apply_static: V tiles for up to STATIC_APPLY_BLOCKS
+// row blocks of one projection, in device memory that exists from module
+// load to process exit (no allocation at run time).
+__device__ __align__(256) uint16_t g_static_vext[STATIC_APPLY_BLOCKS * TM * VEXT_COLS];
+
 }  // namespace
 
 size_t apply_smem_bytes() { return SHRINK_SMEM; }
+
+cudaError_t apply_static_workspace(uint16_t **out)
+{
+    // The host-side name of a __device__ array is not a device address:
+    // resolve it once per device, with that device current.
+    static std::mutex mu;
+    static uint16_t *ptr[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ptr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_vext);
+        if (e != cudaSuccess) return e;
+        ptr[dev] = static_cast<uint16_t *>(p);
+    }
+    *out = ptr[dev];
+    return cudaSuccess;
+}
 
 cudaError_t apply_prepare(int device)
 {

@@ -113,4 +113,11 @@ cudaError_t apply_prepare(int device);
 cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream);
 size_t apply_smem_bytes();
 
+// Row blocks the allocation-free apply (salt_lora_apply_static) can hold in
+// its static device scratch: STATIC_APPLY_BLOCKS * TM * VEXT_COLS bf16 = 2 MiB.
+constexpr int STATIC_APPLY_BLOCKS = 64;
+// Device address of that scratch on the current device (resolved once per
+// device with cudaGetSymbolAddress).
+cudaError_t apply_static_workspace(uint16_t **out);
+
 }  // namespace salt

@@ -714,6 +714,65 @@ salt_status salt_lora_apply(salt_ctx *ctx, const salt_segments *seg, int32_t lay
     return salt_lora_apply_grouped(ctx, seg, 1, &layer, xs, ys, stream);
 }
 
+// Allocation-free variant of salt_lora_apply: the V tiles between the two
+// kernels live in a static device array of this library instead of the
+// segments object's workspace.  See include/salt.h for the contract.
+salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int32_t layer, const void *x, void *y,
+                                   salt_stream_t stream_)
+{
+    if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
+    salt_segments *seg = const_cast<salt_segments *>(seg_);
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (seg->stale) return fail(ctx, SALT_ERR_STALE_SEGMENTS, "a slot named by the segments was reloaded; rebuild");
+    if (layer < 0 || layer >= ctx->n_layers)
+        return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", layer, ctx->n_layers);
+    if (seg->T > 0 && (!x || !y)) return fail(ctx, SALT_ERR_INVALID_ARG, "null x or y");
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15)
+        return fail(ctx, SALT_ERR_ALIGN, "x / y not 16-byte aligned");
+    if (seg->n_blk_bound > STATIC_APPLY_BLOCKS)
+        return fail(ctx, SALT_ERR_TOO_MANY_TOKENS,
+                    "batch may need %d row blocks; the static scratch of salt_lora_apply_static holds %d",
+                    seg->n_blk_bound, STATIC_APPLY_BLOCKS);
+    if (seg->T == 0) return SALT_OK;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    uint16_t *scratch = nullptr;
+    CUDA_OR_FAIL(ctx, apply_static_workspace(&scratch));
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (seg->use_streams.size() > 1 || (seg->use_streams.size() == 1 && seg->use_streams[0] != stream))
+        CUDA_OR_FAIL(ctx, wait_for_uses(seg, stream));
+    add_stream(seg->use_streams, stream);
+    ApplyParams p;
+    std::memset(&p, 0, sizeof p);
+    ApplyProj &pr = p.proj[0];
+    pr.x = static_cast<const uint16_t *>(x);
+    pr.y = static_cast<uint16_t *>(y);
+    pr.A = ctx->arenaA ? ctx->arenaA + ctx->a_off[layer] : nullptr;
+    pr.B = ctx->arenaB ? ctx->arenaB + ctx->b_off[layer] : nullptr;
+    pr.res_off = ctx->res_off[layer];
+    pr.d_in = ctx->d_in[layer];
+    pr.d_out = ctx->d_out[layer];
+    p.n_proj = 1;
+    p.n_unit_prefix[0] = 0;
+    p.n_unit_prefix[1] = (pr.d_out + 63) / 64;
+    p.perm = seg->d.perm;
+    p.blk = seg->d.blk;
+    p.counts = seg->d.counts;
+    p.tok_uoff = seg->d.tok_uoff;
+    p.tok_urank = seg->d.tok_urank;
+    p.tok_su = seg->d.tok_su;
+    p.blk_res = seg->d.blk_res;
+    p.rc_max = ctx->rc_max;
+    p.pool = ctx->pool;
+    p.slot_stride = ctx->slot_stride;
+    p.vext = scratch;
+    p.blk_cap = STATIC_APPLY_BLOCKS;
+    p.err = ctx->err_dev;
+    const int cluster = pr.d_in >= 8192 ? 16 : CLUSTER;
+    CUDA_OR_FAIL(ctx, launch_apply(p, seg->n_blk_bound, cluster, !seg->tables_fresh, stream));
+    seg->tables_fresh = false;
+    return SALT_OK;
+}
+
 salt_status salt_get_device_error(salt_ctx *ctx, salt_stream_t stream, uint32_t *flags)
 {
     if (!ctx || !flags) return SALT_ERR_INVALID_ARG;

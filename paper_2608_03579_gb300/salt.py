@@ -74,6 +74,7 @@ _SIGS = {
     "salt_segments_export": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     "salt_lora_apply": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp]),
     "salt_lora_apply_grouped": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
+    "salt_lora_apply_static": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp]),
     "salt_get_device_error": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]),
 }
 for _name, (_res, _args) in _SIGS.items():
@@ -204,6 +205,11 @@ def salt_segments_export(ctx, seg, max_tokens: int) -> dict:
 
 def salt_lora_apply(ctx, seg, layer: int, x, y, stream=None) -> None:
     _check(_lib.salt_lora_apply(ctx, seg, layer, _ptr(x), _ptr(y), _stream(stream)), ctx)
+
+
+def salt_lora_apply_static(ctx, seg, layer: int, x, y, stream=None) -> None:
+    """salt_lora_apply without any device allocation behind it (static scratch)."""
+    _check(_lib.salt_lora_apply_static(ctx, seg, layer, _ptr(x), _ptr(y), _stream(stream)), ctx)
 
 
 def salt_lora_apply_grouped(ctx, seg, layers, xs, ys, stream=None) -> None:
