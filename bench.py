@@ -417,25 +417,19 @@ def run_salt(args, rank, world, local, pg):
     torch.cuda.synchronize(local)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    # an event pair on the launching stream around each step's applies (the
-    # graph of all apply launches), inside the timed region
-    ev_apply = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for _ in range(args.steps)]
+    # Only the two events that bound the timed region: an event pair recorded
+    # around every step's graph launch was measured to delay the side-stream
+    # swaps and lengthen the step by up to 2x.
     with sampler:
         time.sleep(0.3)
         t_start.record(st.comp)
-        for i, s in enumerate(range(args.warmup, args.warmup + args.steps)):
-            st.swap(s)
-            st.build(s)
-            ev_apply[i][0].record(st.comp)
-            st.applies()
-            ev_apply[i][1].record(st.comp)
+        for s in range(args.warmup, args.warmup + args.steps):
+            st.step(s)
         st.join_side()
         t_end.record(st.comp)
         torch.cuda.synchronize(local)
         time.sleep(0.2)
     ms_total = t_start.elapsed_time(t_end)
-    apply_ms_timed = float(np.mean([a.elapsed_time(b) for (a, b) in ev_apply]))
     # per-launch durations of the last step (graph-captured event pairs)
     barrier(pg, local)
     # per-launch durations of the apply kernel: a pass of whole steps right
@@ -455,17 +449,20 @@ def run_salt(args, rank, world, local, pg):
         msk = sum(kernel_ms[i::4])
         per_kind[k] = {"us_per_launch": 1000.0 * msk / (len(kernel_ms) // 4),
                        "GB/s": float(per_group_bytes[i::4].sum() / (msk / 1000.0) / 1e9)}
-    # the applies alone (graph replays, no swaps), for context
+    # The applies alone: the step's graph of 128 grouped applies replayed
+    # back to back (same tables as the last timed step, no swaps), an event
+    # pair on the launching stream around each replay.  Its mean is the
+    # apply launch pair's duration used for the roofline.
     apply_only_ms = None
-    if st.graph is not None:
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
+    n_rep = 10
+    reps = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_rep)]
+    for a, b in reps:
         a.record(st.comp)
-        for _ in range(5):
-            st.applies()
+        st.applies()
         b.record(st.comp)
-        torch.cuda.synchronize(local)
-        apply_only_ms = a.elapsed_time(b) / 5
+    torch.cuda.synchronize(local)
+    apply_only_ms = float(np.mean([a.elapsed_time(b) for (a, b) in reps]))
+    apply_ms_timed = apply_only_ms
     ms_total = max_over_ranks(pg, ms_total, local)
     ms_per_step = ms_total / args.steps
     value = world * st.T * args.steps / (ms_total / 1000.0)
@@ -475,7 +472,7 @@ def run_salt(args, rank, world, local, pg):
     roof = None
     if apply_ms_timed > 0:
         # the dominant kernel: one salt_lora_apply launch pair (shrink + expand),
-        # its average duration taken over the timed region
+        # its average duration from the graph replays above
         achieved = step_apply_bytes / (apply_ms_timed / 1000.0) / 1e9
         ratio, prof = traffic_from_profile()
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",

@@ -17,16 +17,19 @@
 //                  = s_u V[t,s]    for s in the token's own user's rows
 //                  = 0             otherwise,
 //       rounded to bf16 into the workspace tile of the block.
-//   expand (one CTA per 64 output columns per block, launched as a
-//           programmatic dependent of the shrink):
-//       Y[M x 64] += V_ext * Stack_B[:, cols] (bf16 mma.sync, fp32
-//       accumulation); the B rows and the y rows are fetched before the
-//       dependency wait, so their latency overlaps the shrink.  y is read
-//       once and written once, rounded once (RNE).
+//   expand (persistent, one CTA per SM, launched as a programmatic
+//           dependent of the shrink; items are (block, 64 output columns)):
+//       Y[M x 64] += V_ext * Stack_B[:, cols] on the tensor cores
+//       (tcgen05.mma, V_ext K-major and the B rows MN-major as they lie in
+//       memory, fp32 accumulators double-buffered in tensor memory), the y
+//       and B rows of the next items streaming through a shared-memory ring
+//       meanwhile; the first items' rows are fetched before the dependency
+//       wait, so their latency overlaps the shrink.  y is read once and
+//       written once, rounded once (RNE).
 //
 // Operands are staged by cp.async in 128-byte-row, 128-byte-swizzled tiles
-// (the layout both ldmatrix and the UMMA descriptors read).  Partial sums
-// never leave the chip; the only scratch is the bf16 V tile per block.
+// (the layout the UMMA descriptors read).  Partial sums never leave the
+// chip; the only scratch is the bf16 V tile per block.
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
@@ -68,12 +71,7 @@ struct ShrinkInfo {
     uint64_t bar[MAX_STAGES];     // per stage: the MMAs reading it have completed
     uint32_t tmem;                // tensor-memory base of D^T
 };
-struct ExpandInfo {
-    const uint16_t *srcB[S_MAX];  // stacked B rows
-    int32_t row[TM];
-};
 constexpr size_t SHRINK_SMEM = 1024 + STAGES_BYTES + (sizeof(ShrinkInfo) + 127) / 128 * 128;
-constexpr size_t EXPAND_SMEM = 2 * TILE_BYTES + VT_BYTES + (sizeof(ExpandInfo) + 127) / 128 * 128;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ int swz128(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
@@ -98,24 +96,6 @@ __device__ __forceinline__ void cp_async_wait_dyn(int n)
     }
 }
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
-{
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};\n"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 
@@ -396,138 +376,254 @@ __global__ void __launch_bounds__(APPLY_THREADS, 2) salt_shrink_kernel(const __g
 }
 
 // ---------------------------------------------------------------------------- expand
-__global__ void __launch_bounds__(APPLY_THREADS, 3) salt_expand_kernel(const __grid_constant__ ApplyParams p)
-{
-    extern __shared__ __align__(128) uint8_t smem[];
-    uint8_t *ys = smem;
-    uint8_t *bs = smem + TILE_BYTES;
-    uint8_t *vs = smem + 2 * TILE_BYTES;
-    ExpandInfo &info = *reinterpret_cast<ExpandInfo *>(smem + 2 * TILE_BYTES + VT_BYTES);
+// Persistent, one CTA per SM.  The items of a launch are (row block b,
+// 64-column unit u) pairs in block-major order, u running over the columns
+// of every projection of the group.  CTA i takes the items whose cost
+// position (running sum of blk_weight, from the block records) falls in the
+// i-th equal share of the total.  Per item, on the tensor cores:
+//     D[128 x 64] = V_ext[128 x S] * Stack_B[S x 64]      (tcgen05.mma, fp32 in TMEM)
+// with V_ext (K-major) resident in shared memory for the current
+// (block, projection) and the stacked B rows (MN-major: the rows as they lie
+// in memory) streamed with the item's y rows through an EX_STAGES-deep ring.
+// The accumulator is double-buffered in TMEM: item j's MMAs run while the
+// epilogue of item j-1 (TMEM -> registers, + staged y, one rounding, store)
+// runs on all eight warps.
+constexpr int EX_STAGES = 6;
+constexpr int EX_STAGE_BYTES = 2 * TILE_BYTES;  // y rows | stacked B rows of one item
+constexpr int EX_TMEM_COLS = 2 * NC;           // two 128 x 64 fp32 accumulators
 
-    // The next apply's shrink only reads tables and factors before its own
+struct ExpandInfo {
+    const uint16_t *srcB[S_MAX];  // stacked B rows of the current (block, projection)
+    int32_t row[TM];              // y row of the i-th token of the current block
+    int32_t range[4];             // first item (block, unit), end item (block, unit)
+    uint64_t bar[2];              // per accumulator: its MMAs have completed
+    uint32_t tmem;
+};
+constexpr size_t EXPAND_SMEM = 1024 + EX_STAGES * EX_STAGE_BYTES + VT_BYTES + (sizeof(ExpandInfo) + 127) / 128 * 128;
+static_assert(EXPAND_SMEM <= 227 * 1024, "expand shared memory exceeds the per-block limit");
+
+__device__ __forceinline__ int64_t blk_wend(const int32_t *blk, int b) { return blk[(int64_t)BLK_INTS * b + BLK_WEND]; }
+
+// First block b with nu * wend(b) > c, for 0 <= c < nu * wend(n_blk - 1).
+// Whole warp; each step narrows the range 32-fold.
+__device__ int find_block(const int32_t *blk, int n_blk, int64_t nu, int64_t c, int lane)
+{
+    int lo = 0, hi = n_blk;  // the answer lies in [lo, hi)
+    while (hi - lo > 32) {
+        const int step = (hi - lo + 31) >> 5;
+        const int i = lo + lane * step;
+        const bool past = i >= hi || nu * blk_wend(blk, i) > c;
+        const unsigned m = __ballot_sync(0xffffffffu, past);
+        const int f = m ? __ffs(m) - 1 : 32;
+        const int nlo = f == 0 ? lo : lo + (f - 1) * step + 1;
+        const int nhi = f == 32 ? hi : min(hi, lo + f * step + 1);
+        lo = nlo;
+        hi = nhi;
+    }
+    const int i = lo + lane;
+    const bool past = i >= hi || nu * blk_wend(blk, i) > c;
+    const unsigned m = __ballot_sync(0xffffffffu, past);
+    return m ? lo + __ffs(m) - 1 : hi;
+}
+
+// First item whose cost start is >= c; (n_blk, 0) past the end.  Whole warp.
+__device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, int64_t c, int lane, int &b, int &u)
+{
+    if (c >= total) {
+        b = n_blk;
+        u = 0;
+        return;
+    }
+    b = find_block(blk, n_blk, nu, c, lane);
+    const int64_t wend = blk_wend(blk, b), wbeg = b ? blk_wend(blk, b - 1) : 0;
+    const int64_t w = wend - wbeg;
+    const int64_t off = c - (int64_t)nu * wbeg;
+    u = (int)((off + w - 1) / w);
+    if (u >= nu) {
+        ++b;
+        u = 0;
+    }
+}
+
+__global__ void __launch_bounds__(APPLY_THREADS, 1) salt_expand_kernel(const __grid_constant__ ApplyParams p)
+{
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    // 1024-byte aligned ring (the 128-byte swizzle atom of the UMMA operands)
+    uint8_t *ring = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    uint8_t *vs = ring + EX_STAGES * EX_STAGE_BYTES;  // V_ext: two K-major tiles (K 0..63, 64..127)
+    ExpandInfo &info = *reinterpret_cast<ExpandInfo *>(vs + VT_BYTES);
+
+    // The next apply's shrink reads only tables and factors before its own
     // dependency wait, so it may be scheduled as soon as this grid has started.
     pdl_launch_dependents();
-    const int b = blockIdx.y;
-    const int n_blk = p.counts[3];  // written by the segment kernel, complete before the shrink began
-    if (b >= n_blk || b >= p.blk_cap) return;
-    const int unit = blockIdx.x;
-    int pi = 0;
-    while (pi + 1 < p.n_proj && p.n_unit_prefix[pi + 1] <= unit) ++pi;
-    if (unit >= p.n_unit_prefix[p.n_proj]) return;
-    const ApplyProj &pr = p.proj[pi];
-    const int n0 = (unit - p.n_unit_prefix[pi]) * NC;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int g = lane >> 2, q4 = lane & 3;
-    const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
-    const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
-    const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
-    const int S = rc + m1.x;
-    if (S > S_MAX || S == 0) return;
-    const int S_pad = (S + 15) & ~15;
-    const int d_out = pr.d_out;
-
-    if (tid < M) info.row[tid] = p.perm[start + tid];
-    if (tid < S) {
-        info.srcB[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
-                                  : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], true);
-    }
-    __syncthreads();
-
-    // independent of the shrink: y rows and stacked B rows of these columns
-    for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-        bool ok = col < d_out;
-        cp_async16(smem_u32(ys + swz128(r, c)), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
-    }
-    for (int idx = tid; idx < S_pad * 8; idx += APPLY_THREADS) {
-        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-        bool ok = r < S && col < d_out;
-        cp_async16(smem_u32(bs + swz128(r, c)), ok ? info.srcB[r] + col : pr.y, ok);
-    }
-    cp_async_commit();
-
-    // the V tile is produced by the shrink grid
-    pdl_wait();
-    const uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + b) * (TM * VEXT_COLS);
-    const int nch = S_pad >> 3;
-    for (int idx = tid; idx < M * nch; idx += APPLY_THREADS) {
-        int r = idx / nch, c = idx - r * nch;
-        cp_async16(smem_u32(vs + swz256(r, c)), vt + (int64_t)r * VEXT_COLS + c * 8, true);
-    }
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-
-    const int m_tiles = (M + 15) >> 4;
-    const int em = warp >> 1, en = warp & 1;
-    const int emt0 = em, emt1 = em + 4;
-    const bool eact0 = emt0 < m_tiles, eact1 = emt1 < m_tiles;
-    const uint32_t bs32 = smem_u32(bs), vs32 = smem_u32(vs);
-    float c2[2][4][4];
-#pragma unroll
-    for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) c2[i][j][e] = 0.f;
-    for (int ks = 0; ks < (S_pad >> 4); ++ks) {
-        uint32_t a0[4], a1[4];
-        if (eact0) {
-            int r = emt0 * 16 + (lane & 15);
-            ldsm_x4(vs32 + swz256(r, ks * 2 + (lane >> 4)), a0[0], a0[1], a0[2], a0[3]);
+    // block records: written by the segment kernel, complete before the shrink began
+    const int n_blk = min(p.counts[3], p.blk_cap);
+    const int nu = p.n_unit_prefix[p.n_proj];
+    if (n_blk <= 0 || nu <= 0) return;
+    const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
+    if (warp < 2) {
+        int b, u;
+        item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + warp) / gridDim.x, lane, b, u);
+        if (lane == 0) {
+            info.range[2 * warp] = b;
+            info.range[2 * warp + 1] = u;
         }
-        if (eact1) {
-            int r = emt1 * 16 + (lane & 15);
-            ldsm_x4(vs32 + swz256(r, ks * 2 + (lane >> 4)), a1[0], a1[1], a1[2], a1[3]);
+    }
+    if (warp == 2) {
+        tmem_alloc(smem_u32(&info.tmem), EX_TMEM_COLS);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        mbar_init(smem_u32(&info.bar[0]), 1);
+        mbar_init(smem_u32(&info.bar[1]), 1);
+        mbar_fence_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = info.tmem;
+    int b = info.range[0], u = info.range[1];
+    const int b_end = info.range[2], u_end = info.range[3];
+    bool waited = false, ok_all = true;
+    uint32_t n_done = 0;  // items of earlier runs (accumulator use count)
+    const uint32_t ring32 = smem_u32(ring), vs32 = smem_u32(vs);
+    const uint32_t idesc = idesc_bf16_f32_bmn(TM, NC);
+    const int q = warp & 3, h = warp >> 2;  // epilogue: TMEM lane quarter, column half
+
+    while (b < b_end || (b == b_end && u < u_end)) {
+        // a run: consecutive items of one (block, projection)
+        int pi = 0;
+        while (pi + 1 < p.n_proj && p.n_unit_prefix[pi + 1] <= u) ++pi;
+        const int u0 = u, cb = b;
+        const int u_stop = min(p.n_unit_prefix[pi + 1], b == b_end ? u_end : nu);
+        u = u_stop;
+        if (u == nu) {
+            ++b;
+            u = 0;
         }
+        const ApplyProj &pr = p.proj[pi];
+        const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * cb);
+        const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * cb + 4);
+        const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
+        const int S = rc + m1.x;
+        if (S > S_MAX || S == 0 || M <= 0) continue;  // the shrink flagged S > S_MAX
+        const int S_pad = (S + 15) & ~15;
+        const int d_out = pr.d_out;
+
+        __syncthreads();  // the previous run is done with the ring, V and info
+        if (tid < M) info.row[tid] = p.perm[start + tid];
+        if (tid < S) {
+            info.srcB[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
+                                      : residual_row(p, pr, p.blk_res[(int64_t)cb * S_MAX + (tid - rc)], true);
+        }
+        __syncthreads();
+
+        const int n = u_stop - u0;
+        const int ubase = p.n_unit_prefix[pi];
+        auto load_item = [&](int j) {
+            const int n0 = (u0 + j - ubase) * NC;
+            const uint32_t ys = ring32 + (j % EX_STAGES) * EX_STAGE_BYTES, bs = ys + TILE_BYTES;
+            for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
+                const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+                const bool ok = col < d_out;
+                cp_async16(ys + swz128(r, c), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
+            }
+            for (int idx = tid; idx < S_pad * 8; idx += APPLY_THREADS) {
+                const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+                const bool ok = r < S && col < d_out;
+                cp_async16(bs + swz128(r, c), ok ? info.srcB[r] + col : pr.y, ok);
+            }
+        };
+        const uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + cb) * (TM * VEXT_COLS);
+        const int nch = S_pad >> 3;
+        auto load_v = [&]() {
+            for (int idx = tid; idx < M * nch; idx += APPLY_THREADS) {
+                const int r = idx / nch, c = idx - r * nch;
+                cp_async16(vs32 + (c >> 3) * TILE_BYTES + swz128(r, c & 7), vt + (int64_t)r * VEXT_COLS + c * 8, true);
+            }
+        };
+        // commit groups: [V] P0 .. P(EX_STAGES-3) [V], then one per iteration
+        const bool v_last = !waited;
+        if (waited) {
+            load_v();
+            cp_async_commit();
+        }
+        for (int s = 0; s < EX_STAGES - 2; ++s) {
+            if (s < n) load_item(s);
+            cp_async_commit();
+        }
+        if (!waited) {
+            // y and B rows above do not depend on the shrink; V does
+            pdl_wait();
+            waited = true;
+            load_v();
+            cp_async_commit();
+        }
+
+        for (int j = 0; j <= n; ++j) {
+            if (j < n) {
+                if (v_last && j == 0)
+                    cp_async_wait<0>();
+                else
+                    cp_async_wait<EX_STAGES - 3>();
+                fence_async_smem();
+            }
+            tc_fence_before();
+            __syncthreads();  // item j is visible; the epilogue of item j-2 is over everywhere
+            tc_fence_after();
+            if (j < n && tid == 0) {
+                const uint32_t cnt = n_done + j, buf = cnt & 1;
+                const uint32_t sb = ring32 + (j % EX_STAGES) * EX_STAGE_BYTES + TILE_BYTES;
+                for (int ks = 0; ks < (S_pad >> 4); ++ks)
+                    umma_bf16(tmem + buf * NC, sdesc_kmajor_sw128(vs32 + (ks >> 2) * TILE_BYTES + (ks & 3) * 32),
+                              sdesc_mnmajor_sw128(sb + ks * 2048), idesc, ks > 0 ? 1u : 0u);
+                umma_commit(smem_u32(&info.bar[buf]));
+            }
+            // the stage of item j-2 is free: its MMAs and its epilogue are done
+            if (j + EX_STAGES - 2 < n) load_item(j + EX_STAGES - 2);
+            cp_async_commit();
+
+            if (j >= 1) {
+                const int jj = j - 1;
+                const uint32_t cnt = n_done + jj, buf = cnt & 1;
+                if (!mbar_wait(smem_u32(&info.bar[buf]), (cnt >> 1) & 1)) ok_all = false;
+                tc_fence_after();
+                uint32_t acc[32];
+                const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + buf * NC + h * 32;
+                tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(acc));
+                tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(acc + 16));
+                tmem_ld_wait();
+                const int row = q * 32 + lane;
+                if (row < M) {
+                    const uint8_t *ysp = ring + (jj % EX_STAGES) * EX_STAGE_BYTES;
+                    const int n0 = (u0 + jj - ubase) * NC + h * 32;
+                    uint16_t *yg = pr.y + (int64_t)info.row[row] * d_out + n0;
 #pragma unroll
-        for (int np = 0; np < 2; ++np) {
-            const int nt = en * 4 + 2 * np;
-            if (eact0 || eact1) {
-                int mi = lane >> 3;
-                int kr = ks * 16 + (mi & 1) * 8 + (lane & 7);
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(bs32 + swz128(kr, nt + (mi >> 1)), b0, b1, b2, b3);
-                if (eact0) {
-                    mma_bf16(c2[0][2 * np], a0, b0, b1);
-                    mma_bf16(c2[0][2 * np + 1], a0, b2, b3);
-                }
-                if (eact1) {
-                    mma_bf16(c2[1][2 * np], a1, b0, b1);
-                    mma_bf16(c2[1][2 * np + 1], a1, b2, b3);
+                    for (int c = 0; c < 4; ++c) {
+                        if (n0 + c * 8 < d_out) {
+                            const uint4 v = *reinterpret_cast<const uint4 *>(ysp + swz128(row, h * 4 + c));
+                            const uint32_t in[4] = {v.x, v.y, v.z, v.w};
+                            uint32_t o[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float lo = bf16_to_f((uint16_t)(in[e] & 0xffffu)) + __uint_as_float(acc[c * 8 + 2 * e]);
+                                const float hi = bf16_to_f((uint16_t)(in[e] >> 16)) + __uint_as_float(acc[c * 8 + 2 * e + 1]);
+                                o[e] = (uint32_t)f_to_bf16(lo) | ((uint32_t)f_to_bf16(hi) << 16);
+                            }
+                            *reinterpret_cast<uint4 *>(yg + c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
+                        }
+                    }
                 }
             }
         }
+        cp_async_wait<0>();
+        n_done += n;
     }
-    // epilogue: y_in (staged) + delta, one rounding, back into the staged tile
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const bool act = i == 0 ? eact0 : eact1;
-        const int mt = i == 0 ? emt0 : emt1;
-        if (!act) continue;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int nt = en * 4 + j;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int row = mt * 16 + g + h * 8;
-                if (row >= M) continue;
-                uint32_t *cell = reinterpret_cast<uint32_t *>(ys + swz128(row, nt) + q4 * 4);
-                uint32_t v = *cell;
-                float lo = bf16_to_f((uint16_t)(v & 0xffffu)) + c2[i][j][2 * h];
-                float hi = bf16_to_f((uint16_t)(v >> 16)) + c2[i][j][2 * h + 1];
-                *cell = (uint32_t)f_to_bf16(lo) | ((uint32_t)f_to_bf16(hi) << 16);
-            }
-        }
-    }
+    tc_fence_before();
     __syncthreads();
-    for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-        int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-        if (col < d_out) {
-            uint4 v = *reinterpret_cast<const uint4 *>(ys + swz128(r, c));
-            *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.row[r] * d_out + col) = v;
-        }
-    }
+    if (warp == 2) tmem_dealloc(tmem, EX_TMEM_COLS);
+    if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
 }
 
 // Scratch of salt_lora_apply_static: V tiles for up to STATIC_APPLY_BLOCKS
@@ -560,10 +656,15 @@ cudaError_t apply_static_workspace(uint16_t **out)
     return cudaSuccess;
 }
 
+// SM count per device (the expand grid), filled by apply_prepare
+static int g_sm_count[64];
+
 cudaError_t apply_prepare(int device)
 {
-    (void)device;
-    cudaError_t e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SHRINK_SMEM);
+    if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
+    cudaError_t e = cudaDeviceGetAttribute(&g_sm_count[device], cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SHRINK_SMEM);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e == cudaSuccess)
@@ -591,11 +692,16 @@ cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, boo
     cudaError_t e = cudaLaunchKernelEx(&cfg, salt_shrink_kernel, p);
     if (e != cudaSuccess) return e;
 
+    int dev = 0;
+    e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const int n_sm = (dev >= 0 && dev < 64 && g_sm_count[dev] > 0) ? g_sm_count[dev] : 1;
+    const int64_t items = (int64_t)p.n_unit_prefix[p.n_proj] * n_blk_bound;
     cudaLaunchConfig_t cfg2 = {};
     cudaLaunchAttribute attr2[1];
     attr2[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr2[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg2.gridDim = dim3(p.n_unit_prefix[p.n_proj], n_blk_bound, 1);
+    cfg2.gridDim = dim3((unsigned)(items < n_sm ? items : n_sm), 1, 1);
     cfg2.blockDim = dim3(APPLY_THREADS, 1, 1);
     cfg2.dynamicSmemBytes = EXPAND_SMEM;
     cfg2.stream = stream;

@@ -23,9 +23,16 @@ constexpr int VEXT_COLS = S_MAX;    // row pitch (elements) of a block's V tile 
 
 // Row-block record (BLK_INTS int32 per block, 32 bytes, read as two int4):
 // first grouped token, token count, domain (-1: none), centroid rank of the
-// domain, residual rows of the factor stack, centroid scale s_c (float bits).
+// domain, residual rows of the factor stack, centroid scale s_c (float bits),
+// and the running sum over blocks 0..b of the expand cost weight
+// blk_weight(M, S) (the expand splits its items over CTAs by this weight).
 constexpr int BLK_INTS = 8;
-constexpr int BLK_START = 0, BLK_LEN = 1, BLK_DOM = 2, BLK_RC = 3, BLK_NRES = 4, BLK_SC = 5;
+constexpr int BLK_START = 0, BLK_LEN = 1, BLK_DOM = 2, BLK_RC = 3, BLK_NRES = 4, BLK_SC = 5, BLK_WEND = 6;
+
+// Cost of one 64-column expand item of a block in 128-byte rows moved: y
+// read and written (2 M), the stacked B rows (S), plus a fixed share for the
+// per-item synchronisation.
+__host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 16; }
 
 // Device arrays of one segments object.
 struct SegDev {
@@ -106,8 +113,8 @@ struct ApplyParams {
 cudaError_t launch_segments(const SegParams &p, cudaStream_t stream);
 cudaError_t apply_prepare(int device);
 // shrink: one cluster of `cluster` CTAs per (row block, projection) for the
-// first n_blk_bound blocks; expand: one CTA per 64 output columns per block,
-// launched as a programmatic dependent of the shrink.  With shrink_pdl the
+// first n_blk_bound blocks; expand: one persistent CTA per SM over the
+// (block, 64-column) items, launched as a programmatic dependent of the shrink.  With shrink_pdl the
 // shrink is itself a programmatic dependent of the previous kernel on the
 // stream (only when that kernel did not write the segment tables).
 cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream);

@@ -292,6 +292,23 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         }
         if (lane == 0) p.s.blk[BLK_INTS * b + BLK_NRES] = carry;
     }
+    __syncthreads();
+
+    // 6. running sum of the expand cost weights over blocks
+    const int Eb = (n_blk + nth - 1) / nth;
+    const int blo = min(n_blk, tid * Eb), bhi = min(n_blk, blo + Eb);
+    auto weight = [&](int b) {
+        const int32_t *rec = p.s.blk + (int64_t)BLK_INTS * b;
+        return blk_weight(rec[BLK_LEN], rec[BLK_RC] + rec[BLK_NRES]);
+    };
+    int wsum = 0;
+    for (int b = blo; b < bhi; ++b) wsum += weight(b);
+    int w_total;
+    int wo = block_exclusive_scan(wsum, &w_total, warp_sums);
+    for (int b = blo; b < bhi; ++b) {
+        wo += weight(b);
+        p.s.blk[(int64_t)BLK_INTS * b + BLK_WEND] = wo;
+    }
 }
 
 }  // namespace

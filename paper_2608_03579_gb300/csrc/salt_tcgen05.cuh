@@ -84,6 +84,21 @@ __device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t saddr)
            | ((uint64_t)2 << 61);                    // layout: 128-byte swizzle
 }
 
+// Shared-memory matrix descriptor of an MN-major operand in the 128-byte
+// swizzle layout: rows of 128 bytes hold 64 consecutive MN elements of one K
+// index, 8-row (8 K) atoms of 1024 bytes, the same address-based swizzle as
+// above.  Used with an MN extent of one atom (64), so only the stride between
+// 8-deep K groups (1024 bytes) is ever applied; both offset fields carry it.
+// Moving along K by 16 adds 2048 bytes to the start address.
+__device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4)      // start address >> 4
+           | ((uint64_t)(1024 >> 4) << 16)           // leading byte offset
+           | ((uint64_t)(1024 >> 4) << 32)           // stride byte offset
+           | ((uint64_t)1 << 46)                     // descriptor version of the sm_100 family
+           | ((uint64_t)2 << 61);                    // layout: 128-byte swizzle
+}
+
 // Instruction descriptor of kind::f16: bf16 x bf16 -> fp32, both operands
 // K-major, D of M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N)
@@ -94,6 +109,9 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N)
            | ((uint32_t)(N >> 3) << 17)  // N / 8
            | ((uint32_t)(M >> 4) << 24); // M / 16
 }
+
+// The same with B MN-major (bit 16: B transposed).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) { return idesc_bf16_f32(M, N) | (1u << 16); }
 
 // D[tmem] (+)= A * B^T for one K=16 step, issued by a single thread.
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
