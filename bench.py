@@ -199,19 +199,26 @@ class Step:
         r = self.runner
         if not rank16:
             r.pin_centroids()
-        # initial fill of the whole pool; rank-16 mode reuses 64 distinct blobs
+        # initial fill of the whole pool; rank-16 mode reuses 64 distinct blobs.
+        # The blobs a step swaps in live in one huge-page-backed page-locked
+        # region (salt_host_alloc), as a serving engine's host-side residual
+        # cache would.
         r_slot = 16 if rank16 else 2
         nb = r.blob_bytes(r_slot)
+        pitch = (nb + 255) // 256 * 256
+        n_host = 64 if rank16 else 2 * wl.C4_REGION
+        self.host_buf = salt.salt_host_alloc(n_host * pitch)
+        blob_at = lambda k: self.host_buf.tensor[k * pitch:k * pitch + nb]
         if rank16:
-            base = [r.make_blob(u, 0, r_slot) for u in range(64)]
+            base = [r.make_blob(u, 0, r_slot, out=blob_at(u)) for u in range(64)]
             for u in range(self.w.n_slots):
                 salt.salt_residual_load(r.ctx, u, base[u % 64], None)
             torch.cuda.synchronize()
             self.host_sets = [base, base]
         else:
             r.load_slots()
-            self.host_sets = [[r.make_blob(wl.config4_region(p) + i, 1 + p) for i in range(wl.C4_REGION)]
-                              for p in range(2)]
+            self.host_sets = [[r.make_blob(wl.config4_region(p) + i, 1 + p, out=blob_at(p * wl.C4_REGION + i))
+                               for i in range(wl.C4_REGION)] for p in range(2)]
         self.blob_bytes = nb
         # activations: one contiguous buffer for all projections
         self.x_off, self.y_off = [], []
@@ -314,6 +321,8 @@ class Step:
     def close(self):
         self.graph = None
         self.runner.close()
+        self.host_sets = None
+        self.host_buf.close()
 
 
 # ----------------------------------------------------------------------------- oracle timing
@@ -451,8 +460,8 @@ def run_salt(args, rank, world, local, pg):
                        "GB/s": float(per_group_bytes[i::4].sum() / (msk / 1000.0) / 1e9)}
     # The applies alone: the step's graph of 128 grouped applies replayed
     # back to back (same tables as the last timed step, no swaps), an event
-    # pair on the launching stream around each replay.  Its mean is the
-    # apply launch pair's duration used for the roofline.
+    # pair on the launching stream around each replay.  Its mean over the
+    # 128 launches is the apply kernel's duration used for the roofline.
     apply_only_ms = None
     n_rep = 10
     reps = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_rep)]
@@ -471,14 +480,14 @@ def run_salt(args, rank, world, local, pg):
     # kernel roofline (the apply kernel dominates the step)
     roof = None
     if apply_ms_timed > 0:
-        # the dominant kernel: one salt_lora_apply launch pair (shrink + expand),
+        # the dominant kernel: one salt_apply_kernel launch per grouped apply,
         # its average duration from the graph replays above
         achieved = step_apply_bytes / (apply_ms_timed / 1000.0) / 1e9
         ratio, prof = traffic_from_profile()
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / peaks["hbm_gbs"],
                 "traffic": (ratio * step_apply_bytes / n_launch) if ratio else None,
-                "kernel": "salt_lora_apply_grouped (salt_shrink_kernel + salt_expand_kernel)",
+                "kernel": "salt_apply_kernel (one launch per grouped apply)",
                 "launches_per_step": n_launch,
                 "algorithmic_bytes_per_launch": step_apply_bytes / n_launch,
                 "avg_launch_us": 1000.0 * apply_ms_timed / n_launch,
@@ -553,11 +562,11 @@ def run_salt(args, rank, world, local, pg):
                            "l2": "inputs larger than L2 (the step streams > 8 GB; L2 is 126 MB)",
                            "parallelism": f"replicas x{world}", "launch": "CUDA graph of 128 grouped applies"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": args.steps * (2 * n_launch + 1),
+                "gpu_launches": args.steps * (n_launch + 1),
                 "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
                 "swap_ms_per_step_alone": swap_ms, "apply_only_ms_per_step": apply_only_ms,
                 "apply_kernel_by_group": per_kind,
-                "apply_launch_shape": {k: ctx_info[k] for k in ("cluster_wide", "cluster_size", "apply_smem_bytes",
+                "apply_launch_shape": {k: ctx_info[k] for k in ("apply_ctas", "k_splits_max", "apply_smem_bytes",
                                                                   "block_tokens", "block_users")}}
         print(json.dumps(line), flush=True)
 

@@ -147,9 +147,9 @@ typedef struct salt_ctx_info {
     int64_t arena_bytes;        /* centroid arena, device */
     int64_t pool_bytes;         /* residual slot pool, device */
     int64_t slot_stride;        /* bytes per slot */
-    int32_t cluster_wide;       /* CTAs per shrink cluster when a layer has d_in >= 8192 */
-    int32_t cluster_size;       /* CTAs per shrink cluster otherwise */
-    int32_t apply_smem_bytes;   /* dynamic shared memory per shrink CTA */
+    int32_t apply_ctas;         /* CTAs of one apply launch (one per SM) */
+    int32_t k_splits_max;       /* most d_in splits of one row block's shrink */
+    int32_t apply_smem_bytes;   /* dynamic shared memory per apply CTA */
     int32_t block_tokens;       /* max tokens per row block */
     int32_t block_users;        /* max user runs per row block */
     int32_t reserved;
@@ -182,6 +182,21 @@ int64_t salt_residual_blob_bytes(const salt_config *config, int32_t rank);
 salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, float s_u,
                                     const void *At_u, const void *B_u,
                                     void *blob, int64_t blob_bytes);
+
+/*
+ * Page-locked host memory for residual blobs, backed by transparent huge
+ * pages where the kernel offers them (anonymous mapping rounded up to the
+ * huge-page size, madvise(MADV_HUGEPAGE), every page touched, then
+ * cudaHostRegister).  The host-to-device copies of a swap translate host
+ * addresses page by page; with the base pages of an ordinary pinned
+ * allocation (64 KiB on Arm servers) sustained swapping was measured to
+ * stall for 30-100 ms every few hundred copies, with huge pages not at all.
+ * (The paper has no counterpart; this is a deployment convenience for the
+ * host side of the residual cache.)  Returns NULL on failure; the memory
+ * is zeroed.  Release with salt_host_free (not free or cudaFreeHost).
+ */
+void *salt_host_alloc(int64_t bytes);
+void salt_host_free(void *ptr);
 
 /*
  * Swap a residual into slot `slot` (Section "Multi-Tenant Serving": only
@@ -273,18 +288,19 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
  * this is a deployment convenience of the library.)
  *
  * Same arguments, result and ordering as salt_lora_apply, for one layer.
- * The intermediate V tiles live in a static device array of this library
- * (2 MiB, held by every device that loads the library until the process
- * exits) instead of the segments object's workspace; the call itself
+ * The apply's scratch - the intermediate V tiles, the partial sums of the
+ * split shrink, the per-block ready flags and a launch counter, about
+ * 12 MiB - lives in static device arrays of this library (held by every
+ * device that loads the library until the process exits, zero when it
+ * loads) instead of the segments object's workspace; the call itself
  * allocates nothing.  Limit: the batch may need at most 64 row blocks
  * (blocks hold <= 128 tokens of one domain); a larger batch returns
  * SALT_ERR_TOO_MANY_TOKENS before any device work.  The first call on a
- * device looks up the array's device address (cudaGetSymbolAddress); make
- * that first call before any stream capture.  Every call shares the one
- * array: calls that may overlap on the GPU (on different streams, or from
- * different contexts or threads) race on it and must be serialised by the
- * caller.  Nothing in the array needs to start at zero: each call writes
- * every entry it later reads.
+ * device looks up the arrays' device addresses (cudaGetSymbolAddress);
+ * make that first call before any stream capture.  Every call shares the
+ * one set of arrays: calls that may overlap on the GPU (on different
+ * streams, or from different contexts or threads) race on them and must be
+ * serialised by the caller.
  */
 salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
                                    const void *x, void *y, salt_stream_t stream);

@@ -5,32 +5,41 @@
 // segment builder) concatenates its factors into one stack of
 // S = rc + sum_u r_u rows, [A_c | a_u1 | a_u2 | ...] - the paper's
 // "centroid and residual concatenated into one standard adapter" identity,
-// applied per block - so each block is one dense contraction.  Two kernels:
+// applied per block - so each block is one dense contraction pair.
 //
-//   shrink (one cluster of C CTAs per block and projection; CTA c takes
-//           every C-th 64-wide chunk of d_in):
-//       V^T[S x M] = Stack_A[S x d_in] * X[M x d_in]^T on the tensor cores
+// One persistent kernel per apply, one CTA per SM, in two phases:
+//
+//   shrink units (row block b, projection, K-split s of KS): the unit's
+//       contiguous range of 64-wide d_in chunks streams through a deep
+//       shared-memory ring into the tensor cores,
+//           V^T[S x M] (+)= Stack_A[S x chunk] * X[M x chunk]^T
 //       (tcgen05.mma, fp32 accumulator in tensor memory; the stack is the
-//       128-row operand, the tokens the N = 16..128 operand), partial sums
-//       reduced across the cluster through distributed shared memory, then
-//       V_ext[t,s] = s_c V[t,s]    for s < rc (centroid rows)
-//                  = s_u V[t,s]    for s in the token's own user's rows
-//                  = 0             otherwise,
-//       rounded to bf16 into the workspace tile of the block.
-//   expand (persistent, one CTA per SM, launched as a programmatic
-//           dependent of the shrink; items are (block, 64 output columns)):
-//       Y[M x 64] += V_ext * Stack_B[:, cols] on the tensor cores
-//       (tcgen05.mma, V_ext K-major and the B rows MN-major as they lie in
-//       memory, fp32 accumulators double-buffered in tensor memory), the y
-//       and B rows of the next items streaming through a shared-memory ring
-//       meanwhile; the first items' rows are fetched before the dependency
-//       wait, so their latency overlaps the shrink.  y is read once and
-//       written once, rounded once (RNE).
+//       128-row operand, the tokens the N = 16..128 operand).  Each token
+//       keeps the centroid columns and its own user's columns.  With KS = 1
+//       the unit writes V_ext directly.  Otherwise every split stores an
+//       fp32 partial, waits (bounded) until all splits of the block have,
+//       and then reduces its own slice of the token rows over the splits in
+//       split order (so the result does not depend on timing), writing
+//           V_ext[t,s] = s_c V[t,s]    for s < rc (centroid rows)
+//                      = s_u V[t,s]    for s in the token's own user's rows
+//                      = 0             otherwise
+//       as bf16.  Each unit then counts its rows as written.
+//   expand items (row block, 64 output columns), cost-balanced over CTAs:
+//       Y[M x 64] += V_ext * Stack_B[:, cols] on the tensor cores (V_ext
+//       K-major, the B rows MN-major as they lie in memory, fp32 accumulators
+//       double-buffered in tensor memory), the y and B rows of the next items
+//       streaming through the ring meanwhile.  A run of items of one block
+//       starts by prefetching its first items, then waits (bounded) until
+//       every row of the block's V tile is written.  y is read once and
+//       written once, rounded once.
+//
+// The arrival counters come in two halves chosen by the parity of a launch
+// counter kept in device memory (the last CTA of a launch advances it); a
+// launch zeroes the half the next launch uses, so graph replays of a launch
+// stay correct.
 //
 // Operands are staged by cp.async in 128-byte-row, 128-byte-swizzled tiles
-// (the layout the UMMA descriptors read).  Partial sums never leave the
-// chip; the only scratch is the bf16 V tile per block.
-#include <cooperative_groups.h>
+// (the layout the UMMA descriptors read).
 #include <cuda_bf16.h>
 
 #include <mutex>
@@ -38,44 +47,48 @@
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
 
-namespace cg = cooperative_groups;
-
 namespace salt {
 namespace {
 
 constexpr int KC = 64;                         // K chunk of the shrink (128-byte rows)
-constexpr int NC = 64;                         // output columns per expand CTA
+constexpr int NC = 64;                         // output columns per expand item
 constexpr int TILE_BYTES = TM * 128;           // 128 rows x 128 B
-constexpr int STAGES_BYTES = 96 * 1024;        // shrink stage ring
-constexpr int MAX_STAGES = 6;
-constexpr int MAX_CLUSTER = 16;
-constexpr int TMEM_COLS = 128;                 // D^T: up to 128 token columns
-constexpr int PW = SALT_MAX_CENTROID_RANK + SALT_MAX_RESIDUAL_RANK;  // compact partial width
-constexpr int P_BYTES = TM * PW * 4;
-constexpr int RED_ROWS = TM / CLUSTER;         // rows each CTA reduces (clusters of >= CLUSTER CTAs)
-constexpr int RED_BYTES = RED_ROWS * PW * 4;
+constexpr int RING_BYTES = 192 * 1024;         // shared-memory ring of both phases
+constexpr int A_MAX_STAGES = 8;
+constexpr int B_MAX_STAGES = 10;               // expand: stages of (y rows | stacked B rows) per item
+constexpr int PRODUCER_WARPS = 3;              // expand roles: producers, one MMA warp, epilogue warps
+constexpr int PRODUCER_THREADS = 32 * PRODUCER_WARPS;
+constexpr int EPI_WARPS = 4;
+static_assert(PRODUCER_WARPS + 1 + EPI_WARPS == APPLY_THREADS / 32, "expand warp roles cover the CTA");
+constexpr int TMEM_COLS = 128;                 // shrink: D^T (<= 128 tokens); expand: 2 x 64 columns
+constexpr int KS_MAX = 16;
 constexpr int VT_ROW = VEXT_COLS * 2;          // bytes per V tile row
 constexpr int VT_BYTES = TM * VT_ROW;
-static_assert(P_BYTES + RED_BYTES <= STAGES_BYTES, "partials must fit in the stage area");
+static_assert(5 * 2 * TILE_BYTES + VT_BYTES <= RING_BYTES, "the expand ring must hold 5 full stages and the V tile");
+static_assert(VT_BYTES <= RING_BYTES, "V staging exceeds the ring");
 static_assert(S_MAX <= 128, "the factor stack is the 128-row UMMA operand");
 
-struct ShrinkInfo {
-    const uint16_t *srcA[S_MAX];  // stacked At rows (element 0 of the row for this layer)
-    int32_t row[TM];              // x row of the i-th token of the block
-    int32_t ucol[TM];             // first stacked row of the token's user, -1: none
+struct FusedInfo {
+    const uint16_t *src[S_MAX];  // stacked rows of the current block: A rows (shrink) or B rows (expand)
+    int32_t row[TM];             // x / y row of the i-th token of the block
+    int32_t ucol[TM];            // first stacked row of the token's user, -1: none
     int32_t urank[TM];
     float usu[TM];
-    int16_t rt0[S_MAX];           // residual stack row -> first token of its user run
-    int16_t rt1[S_MAX];           //                    -> one past the last token
-    int16_t rk[S_MAX];            //                    -> rank index within the user
-    uint64_t bar[MAX_STAGES];     // per stage: the MMAs reading it have completed
-    uint32_t tmem;                // tensor-memory base of D^T
+    int16_t rt0[S_MAX];          // residual stack row -> first token of its user run
+    int16_t rt1[S_MAX];          //                    -> one past the last token
+    int16_t rk[S_MAX];           //                    -> rank index within the user
+    uint64_t bar[A_MAX_STAGES];  // shrink: per stage, its MMAs have completed
+    uint64_t bbar[2 * B_MAX_STAGES + 5];  // expand: full, empty per stage; acc full, acc empty; V full
+    int32_t range[4];            // expand: first item (block, unit), end item (block, unit)
+    uint32_t tmem;
+    uint32_t epoch;
+    int32_t last;
 };
-constexpr size_t SHRINK_SMEM = 1024 + STAGES_BYTES + (sizeof(ShrinkInfo) + 127) / 128 * 128;
+constexpr size_t FUSED_SMEM = 1024 + RING_BYTES + (sizeof(FusedInfo) + 127) / 128 * 128;
+static_assert(FUSED_SMEM <= 227 * 1024, "shared memory exceeds the per-block limit");
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ int swz128(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
-__device__ __forceinline__ int swz256(int row, int chunk) { return row * VT_ROW + ((chunk ^ (row & 7)) << 4); }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid)
 {
@@ -85,25 +98,76 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool v
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-// wait until at most n groups are pending (n in [1, MAX_STAGES - 2])
+// wait until at most n groups are pending (n in [0, 7])
 __device__ __forceinline__ void cp_async_wait_dyn(int n)
 {
     switch (n) {
+    case 0: cp_async_wait<0>(); break;
     case 1: cp_async_wait<1>(); break;
     case 2: cp_async_wait<2>(); break;
     case 3: cp_async_wait<3>(); break;
-    default: cp_async_wait<4>(); break;
+    case 4: cp_async_wait<4>(); break;
+    case 5: cp_async_wait<5>(); break;
+    case 6: cp_async_wait<6>(); break;
+    default: cp_async_wait<7>(); break;
     }
 }
 
+// arrive on the mbarrier once all of this thread's earlier cp.async copies have landed
+__device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar)
+{
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+// barrier among the first n threads of the CTA (n a multiple of 32), id 1..15
+__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory"); }
+
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];\n" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Called by one thread after a CTA barrier: every write the CTA made before
+// the barrier is visible GPU-wide before the counter moves.
+__device__ __forceinline__ void signal_add(uint32_t *c)
+{
+    asm volatile("fence.acq_rel.gpu;\n" ::: "memory");
+    atomicAdd(c, 1u);
+}
+
+// Bounded wait (about a quarter of a second) until the counter reads n.
+__device__ bool wait_count(const uint32_t *c, uint32_t n)
+{
+    for (int i = 0; i < (1 << 22); ++i) {
+        if (ld_acquire(c) == n) return true;
+        __nanosleep(32);
+    }
+    return false;
+}
 
 __device__ __forceinline__ float bf16_to_f(uint16_t h) { return __uint_as_float(((uint32_t)h) << 16); }
 __device__ __forceinline__ uint16_t f_to_bf16(float f)
 {
     __nv_bfloat16 b = __float2bfloat16_rn(f);
     return *reinterpret_cast<uint16_t *>(&b);
+}
+
+// Two bf16 (low half first) plus two fp32 deltas, each sum rounded once to
+// bf16 (round to nearest even), packed the same way.
+__device__ __forceinline__ uint32_t add_bf16x2(uint32_t y2, float d_lo, float d_hi)
+{
+    const float lo = __uint_as_float(y2 << 16) + d_lo;
+    const float hi = __uint_as_float(y2 & 0xffff0000u) + d_hi;
+    const __nv_bfloat162 r = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&r);
 }
 
 // Residual row entry of a block's factor stack -> first element of that row.
@@ -115,292 +179,8 @@ __device__ __forceinline__ const uint16_t *residual_row(const ApplyParams &p, co
     return b_side ? base + (int64_t)rank * pr.d_in + (int64_t)k * pr.d_out : base + (int64_t)k * pr.d_in;
 }
 
-// ---------------------------------------------------------------------------- shrink
-constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
-
-__global__ void __launch_bounds__(APPLY_THREADS, 2) salt_shrink_kernel(const __grid_constant__ ApplyParams p)
-{
-    extern __shared__ __align__(128) uint8_t smem_raw[];
-    // 1024-byte aligned stage ring (the 128-byte swizzle atom of the UMMA operands)
-    uint8_t *stages = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    float *P = reinterpret_cast<float *>(stages);
-    float *RED = reinterpret_cast<float *>(stages + P_BYTES);
-    ShrinkInfo &info = *reinterpret_cast<ShrinkInfo *>(stages + STAGES_BYTES);
-
-    // Before the dependency wait this kernel reads only the segment tables
-    // and the factors: the host launches it as a programmatic dependent only
-    // when the previous kernel on the stream did not write those tables.
-    cg::cluster_group cluster = cg::this_cluster();
-    const int C = (int)cluster.num_blocks();
-    const int crank = (int)cluster.block_rank();
-    const int item = blockIdx.x / C;
-    const int b = item / p.n_proj, pi = item - b * p.n_proj;
-    const int n_blk = p.counts[3];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // every CTA of a cluster takes the same exits, before any cluster barrier
-    if (b >= n_blk || b >= p.blk_cap) {
-        if (b < n_blk && tid == 0 && crank == 0 && pi == 0) atomicOr(p.err, SALT_DEVERR_RANK);
-        pdl_wait();
-        pdl_launch_dependents();
-        return;
-    }
-    const ApplyProj &pr = p.proj[pi];
-    const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
-    const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
-    const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
-    const int S = rc + m1.x;
-    const float s_c = __int_as_float(m1.y);
-    if (S > S_MAX || S == 0) {
-        if (S > S_MAX && tid == 0 && crank == 0) atomicOr(p.err, SALT_DEVERR_RANK);
-        pdl_wait();
-        pdl_launch_dependents();
-        return;
-    }
-    const int d_in = pr.d_in;
-
-    // ---- block setup from the segment tables
-    if (tid < M) {
-        const int t = tid;
-        info.row[t] = p.perm[start + t];
-        const int uo = p.tok_uoff[start + t];
-        const int ur = p.tok_urank[start + t];
-        info.ucol[t] = uo >= 0 ? rc + uo : -1;
-        info.urank[t] = ur;
-        info.usu[t] = p.tok_su[start + t];
-        if (uo >= 0) {
-            const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
-            const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
-            for (int k = 0; k < ur; ++k) {
-                const int s = rc + uo + k;
-                if (s < S_MAX) {
-                    if (head) {
-                        info.rt0[s] = (int16_t)t;
-                        info.rk[s] = (int16_t)k;
-                    }
-                    if (tail) info.rt1[s] = (int16_t)(t + 1);
-                }
-            }
-        }
-    }
-    if (tid < S) {
-        info.srcA[tid] = tid < rc ? pr.A + ((int64_t)d * p.rc_max + tid) * d_in
-                                  : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], false);
-    }
-    if (warp == 0) {
-        tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
-        tmem_relinquish();
-    }
-    if (tid == 0) {
-        for (int s = 0; s < MAX_STAGES; ++s) mbar_init(smem_u32(&info.bar[s]), 1);
-        mbar_fence_init();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = info.tmem;
-
-    // ---- stage geometry: A = the factor stack (always 128 rows: the UMMA M
-    // operand), X = the block's tokens rounded to the 16-row UMMA N step
-    const int m_rows = ((M + 15) >> 4) << 4;
-    const int stage_bytes = TILE_BYTES + m_rows * 128;
-    const int nstage = min(MAX_STAGES, STAGES_BYTES / stage_bytes);
-    const uint32_t ring = smem_u32(stages);
-    const uint32_t idesc = idesc_bf16_f32(128, m_rows);
-
-    // chunks are dealt round-robin over the cluster: at any moment the C CTAs
-    // read adjacent pieces of every row
-    const int nk = (d_in + KC - 1) / KC;
-    const int n_my = nk > crank ? (nk - crank + C - 1) / C : 0;
-
-    // each thread's 16-byte pieces of a chunk, resolved once
-    // piece j of this thread is (row (tid + j*256) / 8, 16-byte chunk tid % 8),
-    // the same for every j, so one column offset serves all pieces
-    const int cb = (tid & 7) * 8;
-    const uint16_t *a_src[MAX_PIECES];
-    const uint16_t *x_src[MAX_PIECES];
-#pragma unroll
-    for (int j = 0; j < MAX_PIECES; ++j) {
-        const int r = (tid + j * APPLY_THREADS) >> 3;
-        a_src[j] = r < S ? info.srcA[r] + cb : nullptr;
-        x_src[j] = r < M ? pr.x + (int64_t)info.row[r] * d_in + cb : nullptr;
-    }
-    auto load_a = [&](int i, int st) {
-        const int k0 = (crank + i * C) * KC;
-        const bool ok = k0 + cb < d_in;
-        const uint32_t base = ring + st * stage_bytes;
-#pragma unroll
-        for (int j = 0; j < MAX_PIECES; ++j) {
-            const int r = (tid + j * APPLY_THREADS) >> 3;
-            if (r < S) cp_async16(base + swz128(r, tid & 7), a_src[j] + (ok ? k0 : 0), ok);
-        }
-    };
-    auto load_x = [&](int i, int st) {
-        const int k0 = (crank + i * C) * KC;
-        const bool ok = k0 + cb < d_in;
-        const uint32_t base = ring + st * stage_bytes + TILE_BYTES;
-#pragma unroll
-        for (int j = 0; j < MAX_PIECES; ++j) {
-            const int r = (tid + j * APPLY_THREADS) >> 3;
-            if (r < M) cp_async16(base + swz128(r, tid & 7), x_src[j] + (ok ? k0 : 0), ok);
-        }
-    };
-
-    // ---- nstage-deep pipeline.  The factor rows of the first chunks are
-    // requested before the dependency wait (no preceding kernel writes them),
-    // x only after it; the first commit group carries those factor rows.
-    bool ok_all = true;
-    for (int s = 0; s < nstage - 1 && s < n_my; ++s) load_a(s, s);
-    pdl_wait();
-    // the expand may start once every CTA has passed the wait: anything it
-    // reads before its own wait (y, B rows) is final by now
-    pdl_launch_dependents();
-    for (int s = 0; s < nstage - 1; ++s) {
-        if (s < n_my) load_x(s, s);
-        cp_async_commit();
-    }
-    for (int it = 0; it < n_my; ++it) {
-        const int st = it % nstage;
-        cp_async_wait_dyn(nstage - 2);
-        fence_async_smem();
-        __syncthreads();
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t sa = ring + st * stage_bytes, sx = sa + TILE_BYTES;
-#pragma unroll
-            for (int kk = 0; kk < KC / 16; ++kk)
-                umma_bf16(tmem, sdesc_kmajor_sw128(sa + kk * 32), sdesc_kmajor_sw128(sx + kk * 32), idesc,
-                          (it > 0 || kk > 0) ? 1u : 0u);
-            umma_commit(smem_u32(&info.bar[st]));
-        }
-        const int nxt = it + nstage - 1;
-        if (nxt < n_my) {
-            // the stage of chunk nxt last held chunk it - 1: its MMAs must be done
-            if (it >= 1 && !mbar_wait(smem_u32(&info.bar[(it - 1) % nstage]), ((it - 1) / nstage) & 1))
-                ok_all = false;
-            load_a(nxt, nxt % nstage);
-            load_x(nxt, nxt % nstage);
-        }
-        cp_async_commit();
-    }
-    cp_async_wait<0>();
-    if (n_my > 0 && !mbar_wait(smem_u32(&info.bar[(n_my - 1) % nstage]), ((n_my - 1) / nstage) & 1))
-        ok_all = false;
-    tc_fence_after();
-    __syncthreads();  // the stage ring becomes the partial-sum area
-
-    // ---- D^T (TMEM lanes = stack rows, columns = tokens) -> compact partials:
-    // the centroid rows for every token, a user's rows for that user's tokens
-    if (warp < 4) {
-        const int s = warp * 32 + lane;
-        int col = -1, t0 = 0, t1 = 0;
-        if (s < rc) {
-            col = s;
-            t1 = M;
-        } else if (s < S) {
-            col = rc + info.rk[s];
-            t0 = info.rt0[s];
-            t1 = info.rt1[s];
-        }
-        for (int cg16 = 0; cg16 < (m_rows >> 4); ++cg16) {
-            uint32_t v[16];
-            if (n_my > 0) {
-                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + cg16 * 16, v);
-                tmem_ld_wait();
-            } else {
-#pragma unroll
-                for (int e = 0; e < 16; ++e) v[e] = 0u;
-            }
-#pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                const int t = cg16 * 16 + e;
-                if (col >= 0 && t >= t0 && t < t1) P[t * PW + col] = __uint_as_float(v[e]);
-            }
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
-    if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
-    cluster.sync();
-
-    // ---- reduce the rows this CTA owns over the cluster, scale, mask, store V_ext.
-    // All peers' float4 pieces are requested before any is summed; the sum
-    // runs in peer order, so the result does not depend on timing.
-    const int S_pad = (S + 15) & ~15;
-    const int r0 = crank * M / C, r1 = (crank + 1) * M / C;
-    constexpr int PW4 = PW / 4;
-    for (int idx = tid; idx < (r1 - r0) * PW4; idx += APPLY_THREADS) {
-        const int rr = idx / PW4, c4 = idx - rr * PW4, row = r0 + rr;
-        if (c4 * 4 < rc + info.urank[row]) {
-            float4 v[MAX_CLUSTER];
-#pragma unroll
-            for (int qq = 0; qq < MAX_CLUSTER; ++qq)
-                if (qq < C)
-                    v[qq] = *reinterpret_cast<const float4 *>(cluster.map_shared_rank(P, qq) + row * PW + c4 * 4);
-            float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-            for (int qq = 0; qq < MAX_CLUSTER; ++qq)
-                if (qq < C) {
-                    s.x += v[qq].x;
-                    s.y += v[qq].y;
-                    s.z += v[qq].z;
-                    s.w += v[qq].w;
-                }
-            *reinterpret_cast<float4 *>(RED + rr * PW + c4 * 4) = s;
-        }
-    }
-    __syncthreads();
-    uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + b) * (TM * VEXT_COLS);
-    const int nch = S_pad >> 3;
-    for (int idx = tid; idx < (r1 - r0) * nch; idx += APPLY_THREADS) {
-        const int rr = idx / nch, c = idx - rr * nch, row = r0 + rr;
-        const int uc = info.ucol[row], ur = info.urank[row];
-        const float us = info.usu[row];
-        uint32_t w[4];
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-            uint16_t v2[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int col = c * 8 + 2 * h + e;
-                float v = 0.f;
-                if (col < rc) v = s_c * RED[rr * PW + col];
-                else if (uc >= 0 && col >= uc && col < uc + ur) v = us * RED[rr * PW + rc + (col - uc)];
-                v2[e] = f_to_bf16(v);
-            }
-            w[h] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
-        }
-        *reinterpret_cast<uint4 *>(vt + (int64_t)row * VEXT_COLS + c * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-    }
-    cluster.sync();  // peers have read this CTA's partials
-}
-
-// ---------------------------------------------------------------------------- expand
-// Persistent, one CTA per SM.  The items of a launch are (row block b,
-// 64-column unit u) pairs in block-major order, u running over the columns
-// of every projection of the group.  CTA i takes the items whose cost
-// position (running sum of blk_weight, from the block records) falls in the
-// i-th equal share of the total.  Per item, on the tensor cores:
-//     D[128 x 64] = V_ext[128 x S] * Stack_B[S x 64]      (tcgen05.mma, fp32 in TMEM)
-// with V_ext (K-major) resident in shared memory for the current
-// (block, projection) and the stacked B rows (MN-major: the rows as they lie
-// in memory) streamed with the item's y rows through an EX_STAGES-deep ring.
-// The accumulator is double-buffered in TMEM: item j's MMAs run while the
-// epilogue of item j-1 (TMEM -> registers, + staged y, one rounding, store)
-// runs on all eight warps.
-constexpr int EX_STAGES = 6;
-constexpr int EX_STAGE_BYTES = 2 * TILE_BYTES;  // y rows | stacked B rows of one item
-constexpr int EX_TMEM_COLS = 2 * NC;           // two 128 x 64 fp32 accumulators
-
-struct ExpandInfo {
-    const uint16_t *srcB[S_MAX];  // stacked B rows of the current (block, projection)
-    int32_t row[TM];              // y row of the i-th token of the current block
-    int32_t range[4];             // first item (block, unit), end item (block, unit)
-    uint64_t bar[2];              // per accumulator: its MMAs have completed
-    uint32_t tmem;
-};
-constexpr size_t EXPAND_SMEM = 1024 + EX_STAGES * EX_STAGE_BYTES + VT_BYTES + (sizeof(ExpandInfo) + 127) / 128 * 128;
-static_assert(EXPAND_SMEM <= 227 * 1024, "expand shared memory exceeds the per-block limit");
+// K-split s of KS over nk chunks: [nk * s / KS, nk * (s + 1) / KS)
+__device__ __forceinline__ int split_lo(int nk, int s, int KS) { return (int)((int64_t)nk * s / KS); }
 
 __device__ __forceinline__ int64_t blk_wend(const int32_t *blk, int b) { return blk[(int64_t)BLK_INTS * b + BLK_WEND]; }
 
@@ -426,7 +206,7 @@ __device__ int find_block(const int32_t *blk, int n_blk, int64_t nu, int64_t c, 
     return m ? lo + __ffs(m) - 1 : hi;
 }
 
-// First item whose cost start is >= c; (n_blk, 0) past the end.  Whole warp.
+// First expand item whose cost start is >= c; (n_blk, 0) past the end.  Whole warp.
 __device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, int64_t c, int lane, int &b, int &u)
 {
     if (c >= total) {
@@ -445,22 +225,33 @@ __device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, in
     }
 }
 
-__global__ void __launch_bounds__(APPLY_THREADS, 1) salt_expand_kernel(const __grid_constant__ ApplyParams p)
+constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
+
+__global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __grid_constant__ ApplyParams p)
 {
     extern __shared__ __align__(128) uint8_t smem_raw[];
     // 1024-byte aligned ring (the 128-byte swizzle atom of the UMMA operands)
     uint8_t *ring = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    uint8_t *vs = ring + EX_STAGES * EX_STAGE_BYTES;  // V_ext: two K-major tiles (K 0..63, 64..127)
-    ExpandInfo &info = *reinterpret_cast<ExpandInfo *>(vs + VT_BYTES);
+    FusedInfo &info = *reinterpret_cast<FusedInfo *>(ring + RING_BYTES);
+    const uint32_t ring32 = smem_u32(ring);
+    uint16_t *Vs = reinterpret_cast<uint16_t *>(ring);  // shrink: V tile staging [TM][VEXT_COLS]
 
-    // The next apply's shrink reads only tables and factors before its own
-    // dependency wait, so it may be scheduled as soon as this grid has started.
+    // Before the dependency wait this kernel reads only the segment tables
+    // and the factors: the host launches it as a programmatic dependent only
+    // when the previous kernel on the stream did not write those tables.
+    // The next kernel may be scheduled as soon as every CTA of this one runs.
     pdl_launch_dependents();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // block records: written by the segment kernel, complete before the shrink began
-    const int n_blk = min(p.counts[3], p.blk_cap);
+    const int n_blk = min(p.counts[3], p.w.blk_cap);
+    if (p.counts[3] > p.w.blk_cap && blockIdx.x == 0 && threadIdx.x == 0) atomicOr(p.err, SALT_DEVERR_RANK);
     const int nu = p.n_unit_prefix[p.n_proj];
-    if (n_blk <= 0 || nu <= 0) return;
+    if (n_blk <= 0 || nu <= 0) return;  // the same for every CTA
+    const int n_bp = n_blk * p.n_proj;
+    int KS = max(1, min(KS_MAX, (int)gridDim.x / n_bp));
+    if (KS > 1 && (int64_t)n_bp * KS > p.w.part_cap) KS = max(1, p.w.part_cap / n_bp);
+    const int n_units = n_bp * KS;
+    const int ua = (int)((int64_t)n_units * blockIdx.x / gridDim.x);
+    const int ub = (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
     const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
     if (warp < 2) {
         int b, u;
@@ -471,26 +262,339 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_expand_kernel(const __g
         }
     }
     if (warp == 2) {
-        tmem_alloc(smem_u32(&info.tmem), EX_TMEM_COLS);
+        tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
         tmem_relinquish();
     }
     if (tid == 0) {
-        mbar_init(smem_u32(&info.bar[0]), 1);
-        mbar_init(smem_u32(&info.bar[1]), 1);
+        for (int i = 0; i < A_MAX_STAGES; ++i) mbar_init(smem_u32(&info.bar[i]), 1);
         mbar_fence_init();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = info.tmem;
+    bool ok_all = true, waited = false;
+    // Once per CTA: wait for the previous kernel on the stream (x and y may be
+    // its outputs), then read this launch's epoch; its parity selects the
+    // half of the counters this launch uses.
+    const int n_pairs = SALT_MAX_GROUP * p.w.blk_cap;
+    auto dep_wait = [&]() {
+        pdl_wait();
+        waited = true;
+        if (tid == 0) info.epoch = *reinterpret_cast<volatile uint32_t *>(p.w.seq);
+        __syncthreads();
+        // the counters of the next launch start from zero (the previous
+        // launch, which used them, is complete)
+        const int nxt = ((info.epoch + 1) & 1) * n_pairs;
+        for (int i = blockIdx.x * APPLY_THREADS + tid; i < n_pairs; i += gridDim.x * APPLY_THREADS) {
+            p.w.arrive[nxt + i] = 0u;
+            p.w.vdone[nxt + i] = 0u;
+        }
+    };
+
+    // ================================================================ shrink units
+    uint32_t a_phase = 0;  // parity of the next completion of each stage barrier
+    for (int unit = ua; unit < ub; ++unit) {
+        const int pair = unit / KS, s = unit - pair * KS;
+        const int b = pair / p.n_proj, pi = pair - b * p.n_proj;
+        const ApplyProj &pr = p.proj[pi];
+        const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
+        const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
+        const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
+        const int S = rc + m1.x;
+        const float s_c = __int_as_float(m1.y);
+        const int d_in = pr.d_in;
+        const int nk = (d_in + KC - 1) / KC;
+        const int c0 = split_lo(nk, s, KS), n_my = split_lo(nk, s + 1, KS) - c0;
+        if (S > S_MAX || S == 0 || M <= 0 || n_my <= 0) {
+            if (S > S_MAX && s == 0 && tid == 0) atomicOr(p.err, SALT_DEVERR_RANK);
+            continue;
+        }
+        __syncthreads();  // the previous unit is done with info and the ring
+        if (tid < M) {
+            const int t = tid;
+            info.row[t] = p.perm[start + t];
+            const int uo = p.tok_uoff[start + t];
+            const int ur = p.tok_urank[start + t];
+            info.ucol[t] = uo >= 0 ? rc + uo : -1;
+            info.urank[t] = ur;
+            info.usu[t] = p.tok_su[start + t];
+            if (uo >= 0) {
+                const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
+                const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
+                for (int k = 0; k < ur; ++k) {
+                    const int sr = rc + uo + k;
+                    if (sr < S_MAX) {
+                        if (head) {
+                            info.rt0[sr] = (int16_t)t;
+                            info.rk[sr] = (int16_t)k;
+                        }
+                        if (tail) info.rt1[sr] = (int16_t)(t + 1);
+                    }
+                }
+            }
+        }
+        if (tid < S) {
+            info.src[tid] = tid < rc ? pr.A + ((int64_t)d * p.rc_max + tid) * d_in
+                                     : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], false);
+        }
+        __syncthreads();
+
+        // stage geometry: A = the factor stack (the 128-row UMMA M operand; rows
+        // >= S are never read back), X = the block's tokens rounded to the
+        // 16-row UMMA N step
+        const int m_rows = ((M + 15) >> 4) << 4;
+        const int stage_bytes = TILE_BYTES + m_rows * 128;
+        const int nstage = min(A_MAX_STAGES, RING_BYTES / stage_bytes);
+        const uint32_t idesc = idesc_bf16_f32(128, m_rows);
+        // each thread's 16-byte pieces of a chunk: piece j is (row (tid + j*256) / 8,
+        // 16-byte column tid % 8), so one column offset serves all pieces
+        const int cb = (tid & 7) * 8;
+        const uint16_t *a_src[MAX_PIECES];
+        const uint16_t *x_src[MAX_PIECES];
+#pragma unroll
+        for (int j = 0; j < MAX_PIECES; ++j) {
+            const int r = (tid + j * APPLY_THREADS) >> 3;
+            a_src[j] = r < S ? info.src[r] + cb : nullptr;
+            x_src[j] = r < M ? pr.x + (int64_t)info.row[r] * d_in + cb : nullptr;
+        }
+        auto load_a = [&](int i, int st) {
+            const int k0 = (c0 + i) * KC;
+            const bool ok = k0 + cb < d_in;
+            const uint32_t base = ring32 + st * stage_bytes;
+#pragma unroll
+            for (int j = 0; j < MAX_PIECES; ++j) {
+                const int r = (tid + j * APPLY_THREADS) >> 3;
+                if (r < S) cp_async16(base + swz128(r, tid & 7), a_src[j] + (ok ? k0 : 0), ok);
+            }
+        };
+        auto load_x = [&](int i, int st) {
+            const int k0 = (c0 + i) * KC;
+            const bool ok = k0 + cb < d_in;
+            const uint32_t base = ring32 + st * stage_bytes + TILE_BYTES;
+#pragma unroll
+            for (int j = 0; j < MAX_PIECES; ++j) {
+                const int r = (tid + j * APPLY_THREADS) >> 3;
+                if (r < M) cp_async16(base + swz128(r, tid & 7), x_src[j] + (ok ? k0 : 0), ok);
+            }
+        };
+
+        // nstage-deep pipeline; the factor rows of the first chunks are
+        // requested before the dependency wait, x only after it; the first
+        // commit group carries those factor rows
+        for (int st = 0; st < nstage - 1 && st < n_my; ++st) load_a(st, st);
+        if (!waited) dep_wait();
+        for (int st = 0; st < nstage - 1; ++st) {
+            if (st < n_my) load_x(st, st);
+            cp_async_commit();
+        }
+        uint32_t pending = 0;  // stages with a commit not yet waited for
+        for (int it = 0; it < n_my; ++it) {
+            const int st = it % nstage;
+            cp_async_wait_dyn(nstage - 2);
+            fence_async_smem();
+            __syncthreads();
+            if (tid == 0) {
+                tc_fence_after();
+                const uint32_t sa = ring32 + st * stage_bytes, sx = sa + TILE_BYTES;
+#pragma unroll
+                for (int kk = 0; kk < KC / 16; ++kk)
+                    umma_bf16(tmem, sdesc_kmajor_sw128(sa + kk * 32), sdesc_kmajor_sw128(sx + kk * 32), idesc,
+                              (it > 0 || kk > 0) ? 1u : 0u);
+                umma_commit(smem_u32(&info.bar[st]));
+            }
+            pending |= 1u << st;
+            const int nxt = it + nstage - 1;
+            if (nxt < n_my) {
+                // the stage of chunk nxt last held chunk it - 1: its MMAs must be done
+                if (it >= 1) {
+                    const int ps = (it - 1) % nstage;
+                    if (!mbar_wait(smem_u32(&info.bar[ps]), (a_phase >> ps) & 1)) ok_all = false;
+                    a_phase ^= 1u << ps;
+                    pending &= ~(1u << ps);
+                }
+                load_a(nxt, nxt % nstage);
+                load_x(nxt, nxt % nstage);
+            }
+            cp_async_commit();
+        }
+        cp_async_wait<0>();
+        // every commit is waited for exactly once, keeping the parities in step
+        for (int st = 0; st < nstage; ++st)
+            if ((pending >> st) & 1) {
+                if (!mbar_wait(smem_u32(&info.bar[st]), (a_phase >> st) & 1)) ok_all = false;
+                a_phase ^= 1u << st;
+            }
+        tc_fence_after();
+
+        // ---- D^T (TMEM lanes = stack rows, columns = tokens).  Warp w reads
+        // lanes 32 (w % 4) .. + 31 and every other 16-token group.
+        const int q = warp & 3, th = warp >> 2;
+        const int sr = q * 32 + lane;
+        int t0 = 0, t1 = 0, col = -1;  // tokens this stack row serves, its compact column
+        if (sr < rc) {
+            t1 = M;
+            col = sr;
+        } else if (sr < S) {
+            t0 = info.rt0[sr];
+            t1 = info.rt1[sr];
+            col = rc + info.rk[sr];
+        }
+        const int S_pad = (S + 15) & ~15;
+        const int n_ne = min(KS, nk);  // splits with at least one chunk
+        const int64_t pidx = (int64_t)pi * p.w.blk_cap + b;
+        uint16_t *vt = p.w.vext + pidx * (TM * VEXT_COLS);
+        const int nch = S_pad >> 3;
+        if (KS == 1) {
+            // V_ext straight from the accumulator into the staging tile
+            for (int g = th; g < (m_rows >> 4); g += 2) {
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
+                tmem_ld_wait();
+                if (sr < S_pad) {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const int t = g * 16 + e;
+                        if (t < M) {
+                            float val = 0.f;
+                            if (sr < rc) val = s_c * __uint_as_float(v[e]);
+                            else if (t >= t0 && t < t1) val = info.usu[t] * __uint_as_float(v[e]);
+                            Vs[t * VEXT_COLS + sr] = f_to_bf16(val);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncthreads();
+            for (int idx = tid; idx < M * nch; idx += APPLY_THREADS) {
+                const int r = idx / nch, c = idx - r * nch;
+                *reinterpret_cast<uint4 *>(vt + r * VEXT_COLS + c * 8) =
+                    *reinterpret_cast<const uint4 *>(Vs + r * VEXT_COLS + c * 8);
+            }
+        } else {
+            // fp32 partial: token t's centroid columns, then its own user's columns
+            float *P = p.w.part + (int64_t)unit * (TM * PART_COLS);
+            for (int g = th; g < (m_rows >> 4); g += 2) {
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
+                tmem_ld_wait();
+                if (col >= 0) {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const int t = g * 16 + e;
+                        if (t < M && t >= t0 && t < t1) P[t * PART_COLS + col] = __uint_as_float(v[e]);
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncthreads();
+            // every split of the block stores its partial, then each reduces
+            // its own slice of the token rows over all splits, in split order
+            if (tid == 0) {
+                uint32_t *ctr = p.w.arrive + (info.epoch & 1) * n_pairs + pidx;
+                signal_add(ctr);
+                if (!wait_count(ctr, n_ne)) ok_all = false;
+            }
+            __syncthreads();
+            uint32_t ne_mask = 0;  // the non-empty splits
+            for (int s2 = 0; s2 < KS; ++s2)
+                if (nk >= KS || split_lo(nk, s2 + 1, KS) > split_lo(nk, s2, KS)) ne_mask |= 1u << s2;
+            const int si = nk >= KS ? s : c0;  // index among the non-empty splits
+            const int r0 = M * si / n_ne, r1 = M * (si + 1) / n_ne;
+            float *Ps = reinterpret_cast<float *>(ring);  // [r1 - r0][PART_COLS] sums
+            constexpr int PC4 = PART_COLS / 4;
+            for (int idx = tid; idx < (r1 - r0) * PC4; idx += APPLY_THREADS) {
+                const int rr = idx / PC4, c4 = idx - rr * PC4, t = r0 + rr;
+                if (c4 * 4 >= rc + info.urank[t]) continue;
+                float4 v[KS_MAX];
+                const float *src = p.w.part + ((int64_t)pair * KS * TM + t) * PART_COLS + c4 * 4;
+#pragma unroll
+                for (int s2 = 0; s2 < KS_MAX; ++s2) {
+                    v[s2] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if ((ne_mask >> s2) & 1)
+                        v[s2] = __ldcg(reinterpret_cast<const float4 *>(src + (int64_t)s2 * (TM * PART_COLS)));
+                }
+                float4 acc = v[0];
+#pragma unroll
+                for (int s2 = 1; s2 < KS_MAX; ++s2) {
+                    acc.x += v[s2].x;
+                    acc.y += v[s2].y;
+                    acc.z += v[s2].z;
+                    acc.w += v[s2].w;
+                }
+                *reinterpret_cast<float4 *>(Ps + rr * PART_COLS + c4 * 4) = acc;
+            }
+            __syncthreads();
+            for (int idx = tid; idx < (r1 - r0) * nch; idx += APPLY_THREADS) {
+                const int rr = idx / nch, ch = idx - rr * nch, t = r0 + rr;
+                const int uc = info.ucol[t], ur = info.urank[t];
+                const float us = info.usu[t];
+                const float *ps = Ps + rr * PART_COLS;
+                uint32_t w4[4];
+#pragma unroll
+                for (int hh = 0; hh < 4; ++hh) {
+                    uint16_t v2[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int c = ch * 8 + 2 * hh + e;
+                        float val = 0.f;
+                        if (c < rc) val = s_c * ps[c];
+                        else if (uc >= 0 && c >= uc && c < uc + ur) val = us * ps[rc + (c - uc)];
+                        v2[e] = f_to_bf16(val);
+                    }
+                    w4[hh] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
+                }
+                *reinterpret_cast<uint4 *>(vt + t * VEXT_COLS + ch * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+            }
+        }
+        // this unit's rows of the block's V tile are written
+        __syncthreads();
+        if (tid == 0) signal_add(p.w.vdone + (info.epoch & 1) * n_pairs + pidx);
+    }
+    if (!waited) dep_wait();
+    tc_fence_before();
+    __syncthreads();  // the shrink phase is over: ring and tensor memory change hands
+    tc_fence_after();
+    const uint32_t epoch = info.epoch;
+
+    // ================================================================ expand items
+    // Warp roles per run of items of one (block, projection):
+    //   warps 0-2  producers: cp.async of each item's y rows and stacked B
+    //              rows into a stage; each thread's copies complete on the
+    //              stage's "full" barrier; the V tile once per run;
+    //   warp 3     one thread issues the MMAs of an item into one of two
+    //              accumulators and commits them to "acc full" and "empty";
+    //   warps 4-7  epilogue: TMEM lanes 32 (w % 4) .. + 31 (one token row a
+    //              thread), the item's 64 columns: + staged y, one rounding,
+    //              store; then "acc empty" and "empty".
     int b = info.range[0], u = info.range[1];
     const int b_end = info.range[2], u_end = info.range[3];
-    bool waited = false, ok_all = true;
-    uint32_t n_done = 0;  // items of earlier runs (accumulator use count)
-    const uint32_t ring32 = smem_u32(ring), vs32 = smem_u32(vs);
-    const uint32_t idesc = idesc_bf16_f32_bmn(TM, NC);
-    const int q = warp & 3, h = warp >> 2;  // epilogue: TMEM lane quarter, column half
-
+    uint8_t *vs = ring + RING_BYTES - VT_BYTES;  // V_ext: two K-major tiles (K 0..63, 64..127)
+    const uint32_t vs32 = smem_u32(vs);
+    const uint32_t idesc_b = idesc_bf16_f32_bmn(TM, NC);
+    const uint32_t bb = smem_u32(&info.bbar[0]);
+    auto full_bar = [&](int st) { return bb + 8u * st; };
+    auto empty_bar = [&](int st) { return bb + 8u * (B_MAX_STAGES + st); };
+    auto accf_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + i); };
+    auto acce_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + 2 + i); };
+    const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 4);
+    // The barriers are set up once; their phases run on across runs: item g
+    // (counted over all runs of this CTA) uses slot g % B_MAX_STAGES and
+    // accumulator g & 1, the r-th run's V tile the r-th phase of "V full".
+    if (tid == 0) {
+        for (int st = 0; st < B_MAX_STAGES; ++st) {
+            mbar_init(full_bar(st), PRODUCER_THREADS);
+            mbar_init(empty_bar(st), 1 + EPI_WARPS);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(accf_bar(i), 1);
+            mbar_init(acce_bar(i), EPI_WARPS);
+        }
+        mbar_init(vfull_bar, PRODUCER_THREADS);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    uint32_t g0 = 0, runs = 0;  // items and runs of this CTA so far
     while (b < b_end || (b == b_end && u < u_end)) {
         // a run: consecutive items of one (block, projection)
         int pi = 0;
@@ -507,207 +611,237 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_expand_kernel(const __g
         const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * cb + 4);
         const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
         const int S = rc + m1.x;
-        if (S > S_MAX || S == 0 || M <= 0) continue;  // the shrink flagged S > S_MAX
+        if (S > S_MAX || S == 0 || M <= 0) continue;  // flagged by the shrink phase
         const int S_pad = (S + 15) & ~15;
         const int d_out = pr.d_out;
+        const int n = u_stop - u0;
+        const int ubase = p.n_unit_prefix[pi];
+        // stages sized to this block: y rows rounded to 16, then the stacked
+        // B rows (both parts start on 2048-byte boundaries)
+        const int m_rows = ((M + 15) >> 4) << 4;
+        const int bst = (m_rows + S_pad) * 128;
+        const int nbs = min(B_MAX_STAGES, (RING_BYTES - VT_BYTES) / bst);
 
-        __syncthreads();  // the previous run is done with the ring, V and info
+        // The previous run is over in every role; its MMAs have completed (the
+        // epilogue saw each accumulator full), so the ring may take new rows.
+        __syncthreads();
         if (tid < M) info.row[tid] = p.perm[start + tid];
         if (tid < S) {
-            info.srcB[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
-                                      : residual_row(p, pr, p.blk_res[(int64_t)cb * S_MAX + (tid - rc)], true);
+            info.src[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
+                                     : residual_row(p, pr, p.blk_res[(int64_t)cb * S_MAX + (tid - rc)], true);
         }
         __syncthreads();
 
-        const int n = u_stop - u0;
-        const int ubase = p.n_unit_prefix[pi];
-        auto load_item = [&](int j) {
-            const int n0 = (u0 + j - ubase) * NC;
-            const uint32_t ys = ring32 + (j % EX_STAGES) * EX_STAGE_BYTES, bs = ys + TILE_BYTES;
-            for (int idx = tid; idx < M * 8; idx += APPLY_THREADS) {
-                const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-                const bool ok = col < d_out;
-                cp_async16(ys + swz128(r, c), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
+        if (warp < PRODUCER_WARPS) {
+            auto load_item = [&](int j) {
+                const int n0 = (u0 + j - ubase) * NC;
+                const uint32_t ys = ring32 + (j % nbs) * bst, bs = ys + m_rows * 128;
+                for (int idx = tid; idx < M * 8; idx += PRODUCER_THREADS) {
+                    const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+                    const bool ok = col < d_out;
+                    cp_async16(ys + swz128(r, c), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
+                }
+                for (int idx = tid; idx < S_pad * 8; idx += PRODUCER_THREADS) {
+                    const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+                    const bool ok = r < S && col < d_out;
+                    cp_async16(bs + swz128(r, c), ok ? info.src[r] + col : pr.y, ok);
+                }
+                cp_async_commit();
+                cp_async_arrive_noinc(full_bar((g0 + j) % B_MAX_STAGES));
+            };
+            const int npre = min(n, nbs);
+            for (int j = 0; j < npre; ++j) load_item(j);
+            // V: once every row of the block's tile is written
+            if (tid == 0) {
+                const int n_ne = min(KS, (pr.d_in + KC - 1) / KC);
+                if (!wait_count(p.w.vdone + (epoch & 1) * n_pairs + ((int64_t)pi * p.w.blk_cap + cb), n_ne))
+                    ok_all = false;
             }
-            for (int idx = tid; idx < S_pad * 8; idx += APPLY_THREADS) {
-                const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
-                const bool ok = r < S && col < d_out;
-                cp_async16(bs + swz128(r, c), ok ? info.srcB[r] + col : pr.y, ok);
+            named_sync(1, PRODUCER_THREADS);
+            {
+                const uint16_t *vt = p.w.vext + ((int64_t)pi * p.w.blk_cap + cb) * (TM * VEXT_COLS);
+                const int nch = S_pad >> 3;
+                for (int idx = tid; idx < M * nch; idx += PRODUCER_THREADS) {
+                    const int r = idx / nch, c = idx - r * nch;
+                    cp_async16(vs32 + (c >> 3) * TILE_BYTES + swz128(r, c & 7), vt + (int64_t)r * VEXT_COLS + c * 8, true);
+                }
+                cp_async_commit();
+                cp_async_arrive_noinc(vfull_bar);
             }
-        };
-        const uint16_t *vt = p.vext + ((int64_t)pi * p.blk_cap + cb) * (TM * VEXT_COLS);
-        const int nch = S_pad >> 3;
-        auto load_v = [&]() {
-            for (int idx = tid; idx < M * nch; idx += APPLY_THREADS) {
-                const int r = idx / nch, c = idx - r * nch;
-                cp_async16(vs32 + (c >> 3) * TILE_BYTES + swz128(r, c & 7), vt + (int64_t)r * VEXT_COLS + c * 8, true);
+            for (int j = npre; j < n; ++j) {
+                // the stage last held item j - nbs of this run
+                const uint32_t gp = g0 + j - nbs;
+                if (!mbar_wait(empty_bar(gp % B_MAX_STAGES), (gp / B_MAX_STAGES) & 1)) ok_all = false;
+                load_item(j);
             }
-        };
-        // commit groups: [V] P0 .. P(EX_STAGES-3) [V], then one per iteration
-        const bool v_last = !waited;
-        if (waited) {
-            load_v();
-            cp_async_commit();
-        }
-        for (int s = 0; s < EX_STAGES - 2; ++s) {
-            if (s < n) load_item(s);
-            cp_async_commit();
-        }
-        if (!waited) {
-            // y and B rows above do not depend on the shrink; V does
-            pdl_wait();
-            waited = true;
-            load_v();
-            cp_async_commit();
-        }
-
-        for (int j = 0; j <= n; ++j) {
-            if (j < n) {
-                if (v_last && j == 0)
-                    cp_async_wait<0>();
-                else
-                    cp_async_wait<EX_STAGES - 3>();
-                fence_async_smem();
-            }
-            tc_fence_before();
-            __syncthreads();  // item j is visible; the epilogue of item j-2 is over everywhere
-            tc_fence_after();
-            if (j < n && tid == 0) {
-                const uint32_t cnt = n_done + j, buf = cnt & 1;
-                const uint32_t sb = ring32 + (j % EX_STAGES) * EX_STAGE_BYTES + TILE_BYTES;
-                for (int ks = 0; ks < (S_pad >> 4); ++ks)
-                    umma_bf16(tmem + buf * NC, sdesc_kmajor_sw128(vs32 + (ks >> 2) * TILE_BYTES + (ks & 3) * 32),
-                              sdesc_mnmajor_sw128(sb + ks * 2048), idesc, ks > 0 ? 1u : 0u);
-                umma_commit(smem_u32(&info.bar[buf]));
-            }
-            // the stage of item j-2 is free: its MMAs and its epilogue are done
-            if (j + EX_STAGES - 2 < n) load_item(j + EX_STAGES - 2);
-            cp_async_commit();
-
-            if (j >= 1) {
-                const int jj = j - 1;
-                const uint32_t cnt = n_done + jj, buf = cnt & 1;
-                if (!mbar_wait(smem_u32(&info.bar[buf]), (cnt >> 1) & 1)) ok_all = false;
-                tc_fence_after();
-                uint32_t acc[32];
-                const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + buf * NC + h * 32;
-                tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(acc));
-                tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(acc + 16));
-                tmem_ld_wait();
-                const int row = q * 32 + lane;
-                if (row < M) {
-                    const uint8_t *ysp = ring + (jj % EX_STAGES) * EX_STAGE_BYTES;
-                    const int n0 = (u0 + jj - ubase) * NC + h * 32;
-                    uint16_t *yg = pr.y + (int64_t)info.row[row] * d_out + n0;
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        if (n0 + c * 8 < d_out) {
-                            const uint4 v = *reinterpret_cast<const uint4 *>(ysp + swz128(row, h * 4 + c));
-                            const uint32_t in[4] = {v.x, v.y, v.z, v.w};
-                            uint32_t o[4];
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const float lo = bf16_to_f((uint16_t)(in[e] & 0xffffu)) + __uint_as_float(acc[c * 8 + 2 * e]);
-                                const float hi = bf16_to_f((uint16_t)(in[e] >> 16)) + __uint_as_float(acc[c * 8 + 2 * e + 1]);
-                                o[e] = (uint32_t)f_to_bf16(lo) | ((uint32_t)f_to_bf16(hi) << 16);
-                            }
-                            *reinterpret_cast<uint4 *>(yg + c * 8) = make_uint4(o[0], o[1], o[2], o[3]);
-                        }
-                    }
+            cp_async_wait<0>();
+        } else if (warp == PRODUCER_WARPS) {
+            if (lane == 0) {
+                if (!mbar_wait(vfull_bar, runs & 1)) ok_all = false;
+                for (int j = 0; j < n; ++j) {
+                    const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g & 1;
+                    if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
+                    if (g >= 2 && !mbar_wait(acce_bar(buf), ((g >> 1) - 1) & 1)) ok_all = false;
+                    fence_async_smem();
+                    tc_fence_after();
+                    const uint32_t sb = ring32 + (j % nbs) * bst + m_rows * 128;
+                    for (int ks = 0; ks < (S_pad >> 4); ++ks)
+                        umma_bf16(tmem + buf * NC, sdesc_kmajor_sw128(vs32 + (ks >> 2) * TILE_BYTES + (ks & 3) * 32),
+                                  sdesc_mnmajor_sw128(sb + ks * 2048), idesc_b, ks > 0 ? 1u : 0u);
+                    umma_commit(accf_bar(buf));
+                    umma_commit(empty_bar(slot));
                 }
             }
+            __syncwarp();
+        } else {
+            const int q = warp & 3;
+            const int row = q * 32 + lane;
+            for (int j = 0; j < n; ++j) {
+                const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g & 1;
+                const int st = j % nbs;
+                if (!mbar_wait(accf_bar(buf), (g >> 1) & 1)) ok_all = false;
+                tc_fence_after();
+                uint32_t acc[64];
+                const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + buf * NC;
+#pragma unroll
+                for (int g = 0; g < 4; ++g) tmem_ld16(ta + 16 * g, *reinterpret_cast<uint32_t(*)[16]>(acc + 16 * g));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acce_bar(buf));
+                // the staged y rows of the item (its "full" phase has completed)
+                if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
+                // y + delta, rounded once, back into the staged tile (this
+                // thread's row) ...
+                uint8_t *ysp = ring + st * bst;
+                const int n0 = (u0 + j - ubase) * NC;
+                if (row < M) {
+                    // all loads first: the swizzled cells do not alias, but the
+                    // compiler cannot tell, so interleaved stores would serialise
+                    uint32_t yv[32];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint4 v = *reinterpret_cast<const uint4 *>(ysp + swz128(row, c));
+                        yv[4 * c] = v.x;
+                        yv[4 * c + 1] = v.y;
+                        yv[4 * c + 2] = v.z;
+                        yv[4 * c + 3] = v.w;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        yv[i] = add_bf16x2(yv[i], __uint_as_float(acc[2 * i]), __uint_as_float(acc[2 * i + 1]));
+#pragma unroll
+                    for (int c = 0; c < 8; ++c)
+                        *reinterpret_cast<uint4 *>(ysp + swz128(row, c)) =
+                            make_uint4(yv[4 * c], yv[4 * c + 1], yv[4 * c + 2], yv[4 * c + 3]);
+                }
+                __syncwarp();
+                // ... then the warp's 32 rows go out whole: 8 lanes per
+                // 128-byte row piece, 4 rows per store
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = q * 32 + i * 4 + (lane >> 3), c = lane & 7, col = n0 + c * 8;
+                    if (r < M && col < d_out)
+                        *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.row[r] * d_out + col) =
+                            *reinterpret_cast<const uint4 *>(ysp + swz128(r, c));
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty_bar(slot));
+            }
         }
-        cp_async_wait<0>();
-        n_done += n;
+        g0 += n;
+        ++runs;
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 2) tmem_dealloc(tmem, EX_TMEM_COLS);
+    if (warp == 2) tmem_dealloc(tmem, TMEM_COLS);
     if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
+    // the last CTA to finish advances the epoch (every CTA read it above)
+    if (tid == 0) {
+        __threadfence();
+        const uint32_t done = atomicAdd(p.w.seq + 1, 1u);
+        if (done == gridDim.x - 1) {
+            atomicExch(p.w.seq + 1, 0u);
+            __threadfence();
+            atomicAdd(p.w.seq, 1u);
+        }
+    }
 }
 
-// Scratch of salt_lora_apply_static: V tiles for up to STATIC_APPLY_BLOCKS
-// row blocks of one projection, in device memory that exists from module
-// load to process exit (no allocation at run time).
+// Scratch of salt_lora_apply_static: V tiles, partial tiles, flags and the
+// epoch for up to STATIC_APPLY_BLOCKS row blocks of one projection, in device
+// memory that exists from module load to process exit (no allocation at run
+// time).  Zero-initialised.
 __device__ __align__(256) uint16_t g_static_vext[STATIC_APPLY_BLOCKS * TM * VEXT_COLS];
+__device__ __align__(256) float g_static_part[STATIC_PART_CAP * TM * PART_COLS];
+__device__ __align__(256) uint32_t g_static_arrive[2 * SALT_MAX_GROUP * STATIC_APPLY_BLOCKS];
+__device__ __align__(256) uint32_t g_static_vdone[2 * SALT_MAX_GROUP * STATIC_APPLY_BLOCKS];
+__device__ __align__(256) uint32_t g_static_seq[2];
+
+// SM count per device (the grid of the apply kernel), filled by apply_prepare
+int g_sm_count[64];
 
 }  // namespace
 
-size_t apply_smem_bytes() { return SHRINK_SMEM; }
+size_t apply_smem_bytes() { return FUSED_SMEM; }
 
-cudaError_t apply_static_workspace(uint16_t **out)
+cudaError_t apply_static_workspace(ApplyWork *out)
 {
     // The host-side name of a __device__ array is not a device address:
-    // resolve it once per device, with that device current.
+    // resolve them once per device, with that device current.
     static std::mutex mu;
-    static uint16_t *ptr[64] = {};
+    static ApplyWork ws[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(mu);
-    if (!ptr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_vext);
-        if (e != cudaSuccess) return e;
-        ptr[dev] = static_cast<uint16_t *>(p);
+    if (!ws[dev].vext) {
+        ApplyWork w = {};
+        void *a = nullptr, *b = nullptr, *c = nullptr, *d = nullptr, *f = nullptr;
+        if ((e = cudaGetSymbolAddress(&a, g_static_vext)) != cudaSuccess) return e;
+        if ((e = cudaGetSymbolAddress(&b, g_static_part)) != cudaSuccess) return e;
+        if ((e = cudaGetSymbolAddress(&c, g_static_arrive)) != cudaSuccess) return e;
+        if ((e = cudaGetSymbolAddress(&d, g_static_vdone)) != cudaSuccess) return e;
+        if ((e = cudaGetSymbolAddress(&f, g_static_seq)) != cudaSuccess) return e;
+        w.vext = static_cast<uint16_t *>(a);
+        w.blk_cap = STATIC_APPLY_BLOCKS;
+        w.part = static_cast<float *>(b);
+        w.part_cap = STATIC_PART_CAP;
+        w.arrive = static_cast<uint32_t *>(c);
+        w.vdone = static_cast<uint32_t *>(d);
+        w.seq = static_cast<uint32_t *>(f);
+        ws[dev] = w;
     }
-    *out = ptr[dev];
+    *out = ws[dev];
     return cudaSuccess;
 }
-
-// SM count per device (the expand grid), filled by apply_prepare
-static int g_sm_count[64];
 
 cudaError_t apply_prepare(int device)
 {
     if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
     cudaError_t e = cudaDeviceGetAttribute(&g_sm_count[device], cudaDevAttrMultiProcessorCount, device);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SHRINK_SMEM);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(salt_shrink_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(salt_expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)EXPAND_SMEM);
-    return e;
+    return cudaFuncSetAttribute(salt_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FUSED_SMEM);
 }
 
-cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream)
+cudaError_t launch_apply(const ApplyParams &p, bool pdl, cudaStream_t stream)
 {
-    if (n_blk_bound <= 0) return cudaSuccess;
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = cluster;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
-    cfg.gridDim = dim3(cluster * p.n_proj * n_blk_bound, 1, 1);
-    cfg.blockDim = dim3(APPLY_THREADS, 1, 1);
-    cfg.dynamicSmemBytes = SHRINK_SMEM;
-    cfg.stream = stream;
-    cfg.attrs = attr;
-    cfg.numAttrs = shrink_pdl ? 2 : 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, salt_shrink_kernel, p);
-    if (e != cudaSuccess) return e;
-
     int dev = 0;
-    e = cudaGetDevice(&dev);
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     const int n_sm = (dev >= 0 && dev < 64 && g_sm_count[dev] > 0) ? g_sm_count[dev] : 1;
-    const int64_t items = (int64_t)p.n_unit_prefix[p.n_proj] * n_blk_bound;
-    cudaLaunchConfig_t cfg2 = {};
-    cudaLaunchAttribute attr2[1];
-    attr2[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr2[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg2.gridDim = dim3((unsigned)(items < n_sm ? items : n_sm), 1, 1);
-    cfg2.blockDim = dim3(APPLY_THREADS, 1, 1);
-    cfg2.dynamicSmemBytes = EXPAND_SMEM;
-    cfg2.stream = stream;
-    cfg2.attrs = attr2;
-    cfg2.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg2, salt_expand_kernel, p);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(n_sm, 1, 1);
+    cfg.blockDim = dim3(APPLY_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = FUSED_SMEM;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, salt_apply_kernel, p);
 }
 
 }  // namespace salt

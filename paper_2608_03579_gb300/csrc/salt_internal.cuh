@@ -15,7 +15,6 @@ namespace salt {
 // rows: rc_max + umax * r_max <= S_MAX.
 constexpr int TM = 128;
 constexpr int S_MAX = 128;
-constexpr int CLUSTER = 8;          // CTAs per row block in the shrink (split of d_in)
 constexpr int APPLY_THREADS = 256;
 constexpr int SEG_THREADS = 1024;
 
@@ -31,8 +30,9 @@ constexpr int BLK_START = 0, BLK_LEN = 1, BLK_DOM = 2, BLK_RC = 3, BLK_NRES = 4,
 
 // Cost of one 64-column expand item of a block in 128-byte rows moved: y
 // read and written (2 M), the stacked B rows (S), plus a fixed share for the
-// per-item synchronisation.
-__host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 16; }
+// per-item handoffs between the expand's warp roles (measured at about
+// 0.5 us an item, 128 rows' worth at the per-SM streaming rate).
+__host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 128; }
 
 // Device arrays of one segments object.
 struct SegDev {
@@ -56,13 +56,29 @@ struct SegDev {
     int32_t *blk_res;      // [max_tokens * S_MAX]
 };
 
-// Scratch of the apply path: one V tile (bf16 [TM][VEXT_COLS]) per
-// (projection of a group, row block), written by the shrink kernel and read
-// by the expand kernel of the same launch pair.
+// Scratch of the apply path, owned by a segments object (one apply at a
+// time uses it; applies on different streams are serialised).
+//   vext:   one V tile (bf16 [TM][VEXT_COLS]) per (projection of a group,
+//           row block), written by the shrink phase, read by the expand
+//           phase of the same launch;
+//   part:   fp32 partial V tiles ([TM][PART_COLS]) of the K-split shrink units;
+//   arrive: [2][pairs], per (projection, row block): split partials stored;
+//   vdone:  [2][pairs], per (projection, row block): V row slices written;
+//           a launch uses the half of its epoch's parity and zeroes the
+//           other half for the next launch;
+//   seq:    [0] launch counter (the epoch), [1] CTAs of the running launch
+//           that have finished.
 struct ApplyWork {
     uint16_t *vext;        // [SALT_MAX_GROUP * blk_cap * TM * VEXT_COLS]
     int32_t blk_cap;
+    float *part;           // [part_cap * TM * PART_COLS]
+    int32_t part_cap;
+    uint32_t *arrive;      // [2 * SALT_MAX_GROUP * blk_cap]
+    uint32_t *vdone;       // [2 * SALT_MAX_GROUP * blk_cap]
+    uint32_t *seq;         // [2]
 };
+constexpr int PART_COLS = SALT_MAX_CENTROID_RANK + SALT_MAX_RESIDUAL_RANK;  // centroid | own residual
+constexpr int PART_CAP = 512;  // partial tiles per segments object (20 MiB)
 
 struct SegParams {
     SegDev s;
@@ -104,27 +120,29 @@ struct ApplyParams {
     int32_t rc_max;
     const uint8_t *pool;
     int64_t slot_stride;
-    uint16_t *vext;       // workspace, [n_proj][blk_cap][TM][VEXT_COLS]
-    int32_t blk_cap;
+    ApplyWork w;
     uint32_t *err;
 };
 
 // Kernel launchers (defined next to the kernels).
 cudaError_t launch_segments(const SegParams &p, cudaStream_t stream);
 cudaError_t apply_prepare(int device);
-// shrink: one cluster of `cluster` CTAs per (row block, projection) for the
-// first n_blk_bound blocks; expand: one persistent CTA per SM over the
-// (block, 64-column) items, launched as a programmatic dependent of the shrink.  With shrink_pdl the
-// shrink is itself a programmatic dependent of the previous kernel on the
-// stream (only when that kernel did not write the segment tables).
-cudaError_t launch_apply(const ApplyParams &p, int n_blk_bound, int cluster, bool shrink_pdl, cudaStream_t stream);
+// One persistent CTA per SM: the shrink units (row block, projection,
+// K-split) first, then the expand items (row block, 64 output columns).
+// With pdl the launch is a programmatic dependent of the previous kernel on
+// the stream (only when that kernel did not write the segment tables).
+cudaError_t launch_apply(const ApplyParams &p, bool pdl, cudaStream_t stream);
 size_t apply_smem_bytes();
 
-// Row blocks the allocation-free apply (salt_lora_apply_static) can hold in
-// its static device scratch: STATIC_APPLY_BLOCKS * TM * VEXT_COLS bf16 = 2 MiB.
+// Row blocks and partial tiles the allocation-free apply
+// (salt_lora_apply_static) can use from its static device scratch.
 constexpr int STATIC_APPLY_BLOCKS = 64;
-// Device address of that scratch on the current device (resolved once per
-// device with cudaGetSymbolAddress).
-cudaError_t apply_static_workspace(uint16_t **out);
+// A single-layer apply splits a row block's shrink at most (SMs / blocks)
+// ways, so up to 256 SMs the static partial tiles never bind and the static
+// apply makes the same split as salt_lora_apply.
+constexpr int STATIC_PART_CAP = 256;
+// The static scratch on the current device (addresses resolved once per
+// device with cudaGetSymbolAddress); blk_cap = STATIC_APPLY_BLOCKS.
+cudaError_t apply_static_workspace(ApplyWork *out);
 
 }  // namespace salt

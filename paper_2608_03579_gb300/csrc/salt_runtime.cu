@@ -14,6 +14,10 @@
 #include <string>
 #include <vector>
 #include <algorithm>
+#include <map>
+#include <mutex>
+
+#include <sys/mman.h>
 
 #include "salt_internal.cuh"
 
@@ -207,9 +211,60 @@ cudaError_t wait_for_uses(salt_segments *seg, cudaStream_t stream)
     return cudaSuccess;
 }
 
+// Huge-page size of the kernel's transparent huge pages (2 MiB when unknown).
+int64_t thp_bytes()
+{
+    int64_t v = 0;
+    if (FILE *f = std::fopen("/sys/kernel/mm/transparent_hugepage/hpage_pmd_size", "r")) {
+        long long x = 0;
+        if (std::fscanf(f, "%lld", &x) == 1) v = x;
+        std::fclose(f);
+    }
+    return v > 0 ? v : (int64_t)2 << 20;
+}
+
+std::mutex g_host_mu;
+std::map<void *, size_t> g_host_maps;  // salt_host_alloc regions and their mapped sizes
+
 }  // namespace
 
 extern "C" {
+
+void *salt_host_alloc(int64_t bytes)
+{
+    if (bytes <= 0) return nullptr;
+    const int64_t hp = thp_bytes();
+    const size_t size = (size_t)((bytes + hp - 1) / hp * hp);
+    void *p = mmap(nullptr, size, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+    if (p == MAP_FAILED) return nullptr;
+#ifdef MADV_HUGEPAGE
+    madvise(p, size, MADV_HUGEPAGE);  // advice only: base pages if refused
+#endif
+    std::memset(p, 0, size);  // fault every page in before it is registered
+    if (cudaHostRegister(p, size, cudaHostRegisterDefault) != cudaSuccess) {
+        cudaGetLastError();
+        munmap(p, size);
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(g_host_mu);
+    g_host_maps[p] = size;
+    return p;
+}
+
+void salt_host_free(void *ptr)
+{
+    if (!ptr) return;
+    size_t size = 0;
+    {
+        std::lock_guard<std::mutex> lock(g_host_mu);
+        auto it = g_host_maps.find(ptr);
+        if (it == g_host_maps.end()) return;
+        size = it->second;
+        g_host_maps.erase(it);
+    }
+    cudaHostUnregister(ptr);
+    munmap(ptr, size);
+}
 
 int32_t salt_abi_version(void) { return SALT_ABI_VERSION; }
 
@@ -247,8 +302,13 @@ salt_status salt_ctx_get_info(const salt_ctx *ctx, salt_ctx_info *info)
     info->arena_bytes = (int64_t)ctx->n_domains * ctx->rc_max * (ctx->sum_din + ctx->sum_dout) * 2;
     info->pool_bytes = ctx->slot_stride * (int64_t)ctx->n_slots;
     info->slot_stride = ctx->slot_stride;
-    info->cluster_wide = 16;
-    info->cluster_size = CLUSTER;
+    int dev_sms = 0;
+    if (cudaDeviceGetAttribute(&dev_sms, cudaDevAttrMultiProcessorCount, ctx->device) != cudaSuccess) {
+        cudaGetLastError();
+        dev_sms = 0;
+    }
+    info->apply_ctas = dev_sms;
+    info->k_splits_max = 16;
     info->apply_smem_bytes = (int32_t)apply_smem_bytes();
     info->block_tokens = TM;
     info->block_users = ctx->umax;
@@ -468,8 +528,16 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
               alloc(&seg->d.tok_urank, n) && alloc(reinterpret_cast<int32_t **>(&seg->d.tok_su), n) &&
               alloc(&seg->d.blk_res, (size_t)n * S_MAX);
     seg->work.blk_cap = block_bound_loose(ctx, n);
-    ok = ok && cudaMalloc(&seg->work.vext, (size_t)SALT_MAX_GROUP * seg->work.blk_cap * TM * VEXT_COLS * 2) ==
-                   cudaSuccess;
+    seg->work.part_cap = PART_CAP;
+    const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
+    ok = ok && cudaMalloc(&seg->work.vext, n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
+         cudaMalloc(&seg->work.part, (size_t)PART_CAP * TM * PART_COLS * sizeof(float)) == cudaSuccess &&
+         cudaMalloc(&seg->work.arrive, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
+         cudaMalloc(&seg->work.vdone, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
+         cudaMalloc(&seg->work.seq, 2 * sizeof(uint32_t)) == cudaSuccess &&
+         cudaMemset(seg->work.arrive, 0, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
+         cudaMemset(seg->work.vdone, 0, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
+         cudaMemset(seg->work.seq, 0, 2 * sizeof(uint32_t)) == cudaSuccess;
     for (int i = 0; ok && i < 2; ++i) {
         ok = cudaHostAlloc(&seg->staging[i], 2 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
              cudaEventCreateWithFlags(&seg->staging_ev[i], cudaEventDisableTiming) == cudaSuccess;
@@ -503,6 +571,10 @@ void salt_segments_destroy(salt_segments *seg)
                        seg->d.blk_res};
     for (int32_t *p : arrs) cudaFree(p);
     cudaFree(seg->work.vext);
+    cudaFree(seg->work.part);
+    cudaFree(seg->work.arrive);
+    cudaFree(seg->work.vdone);
+    cudaFree(seg->work.seq);
     for (int i = 0; i < 2; ++i) {
         if (seg->staging[i]) cudaFreeHost(seg->staging[i]);
         if (seg->staging_ev[i]) cudaEventDestroy(seg->staging_ev[i]);
@@ -677,11 +749,10 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
         CUDA_OR_FAIL(ctx, wait_for_uses(seg, stream));
     add_stream(seg->use_streams, stream);
     p.n_proj = n;
-    int units = 0, max_din = 0;
+    int units = 0;
     for (int i = 0; i < n; ++i) {
         p.n_unit_prefix[i] = units;
         units += (p.proj[i].d_out + 63) / 64;
-        max_din = std::max(max_din, p.proj[i].d_in);
     }
     p.n_unit_prefix[n] = units;
     p.perm = seg->d.perm;
@@ -694,14 +765,11 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
     p.rc_max = ctx->rc_max;
     p.pool = ctx->pool;
     p.slot_stride = ctx->slot_stride;
-    p.vext = seg->work.vext;
-    p.blk_cap = seg->work.blk_cap;
+    p.w = seg->work;
     p.err = ctx->err_dev;
-    // wide inputs split d_in over 16 CTAs so each streams a shorter slice
-    const int cluster = max_din >= 8192 ? 16 : CLUSTER;
     // The first apply after a build waits for the segment kernel in full;
     // later ones overlap their table reads with the previous kernel.
-    CUDA_OR_FAIL(ctx, launch_apply(p, seg->n_blk_bound, cluster, !seg->tables_fresh, stream));
+    CUDA_OR_FAIL(ctx, launch_apply(p, !seg->tables_fresh, stream));
     seg->tables_fresh = false;
     return SALT_OK;
 }
@@ -735,7 +803,7 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
                     seg->n_blk_bound, STATIC_APPLY_BLOCKS);
     if (seg->T == 0) return SALT_OK;
     if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
-    uint16_t *scratch = nullptr;
+    ApplyWork scratch;
     CUDA_OR_FAIL(ctx, apply_static_workspace(&scratch));
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
     if (seg->use_streams.size() > 1 || (seg->use_streams.size() == 1 && seg->use_streams[0] != stream))
@@ -764,11 +832,9 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     p.rc_max = ctx->rc_max;
     p.pool = ctx->pool;
     p.slot_stride = ctx->slot_stride;
-    p.vext = scratch;
-    p.blk_cap = STATIC_APPLY_BLOCKS;
+    p.w = scratch;
     p.err = ctx->err_dev;
-    const int cluster = pr.d_in >= 8192 ? 16 : CLUSTER;
-    CUDA_OR_FAIL(ctx, launch_apply(p, seg->n_blk_bound, cluster, !seg->tables_fresh, stream));
+    CUDA_OR_FAIL(ctx, launch_apply(p, !seg->tables_fresh, stream));
     seg->tables_fresh = false;
     return SALT_OK;
 }

@@ -51,7 +51,7 @@ class salt_config(ctypes.Structure):
 
 class salt_ctx_info(ctypes.Structure):
     _fields_ = [("arena_bytes", ctypes.c_int64), ("pool_bytes", ctypes.c_int64), ("slot_stride", ctypes.c_int64),
-                ("cluster_wide", ctypes.c_int32), ("cluster_size", ctypes.c_int32),
+                ("apply_ctas", ctypes.c_int32), ("k_splits_max", ctypes.c_int32),
                 ("apply_smem_bytes", ctypes.c_int32), ("block_tokens", ctypes.c_int32),
                 ("block_users", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
@@ -76,6 +76,8 @@ _SIGS = {
     "salt_lora_apply_grouped": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
     "salt_lora_apply_static": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp]),
     "salt_get_device_error": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]),
+    "salt_host_alloc": (_vp, [_i64]),
+    "salt_host_free": (None, [_vp]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -162,6 +164,45 @@ def salt_residual_blob_pack(d_in, d_out, rank: int, s_u: float, At_u, B_u, blob,
     cfg = make_config(d_in, d_out)
     _check(_lib.salt_residual_blob_pack(ctypes.byref(cfg), rank, float(s_u), _ptr(At_u), _ptr(B_u),
                                         _ptr(blob), blob_bytes))
+
+
+class HostBuffer:
+    """Huge-page-backed page-locked host memory from salt_host_alloc, viewed
+    as a uint8 torch tensor (``.tensor``); freed by ``close()`` or on
+    garbage collection."""
+
+    def __init__(self, nbytes: int):
+        import torch
+        self.ptr = _lib.salt_host_alloc(int(nbytes))
+        if not self.ptr:
+            raise SaltError(2, f"salt_host_alloc({nbytes}) failed")
+        self.nbytes = int(nbytes)
+        arr = np.ctypeslib.as_array((ctypes.c_uint8 * self.nbytes).from_address(self.ptr))
+        self.tensor = torch.from_numpy(arr)
+
+    def close(self):
+        if self.ptr:
+            self.tensor = None
+            _lib.salt_host_free(self.ptr)
+            self.ptr = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def salt_host_alloc(nbytes: int) -> HostBuffer:
+    return HostBuffer(nbytes)
+
+
+def salt_host_free(buf) -> None:
+    """Release a HostBuffer (or a raw pointer from the C call)."""
+    if isinstance(buf, HostBuffer):
+        buf.close()
+    elif buf:
+        _lib.salt_host_free(buf)
 
 
 def salt_residual_load(ctx, slot: int, host_blob, stream=None) -> None:

@@ -46,12 +46,16 @@ def test_config0_tiny(salt_lib, oracle_mod, wl, y_mode):
 
 
 def test_config1_qkv_grouped_and_single(salt_lib, oracle_mod, wl):
+    # A grouped launch may split d_in differently from single launches (the
+    # split depends on how many (block, projection) pairs share the launch),
+    # so the two agree to rounding, each within the tolerance of the oracle.
     w = wl.config1()
     grouped = run_gpu(w, [[0, 1, 2]])
     single = run_gpu(w, [[0], [1], [2]])
     for l in range(3):
-        assert_close(grouped[l], oracle_layer(oracle_mod, w, l), f"config1 layer {l}")
-        np.testing.assert_array_equal(grouped[l], single[l])
+        ref = oracle_layer(oracle_mod, w, l)
+        assert_close(grouped[l], ref, f"config1 layer {l}, grouped")
+        assert_close(single[l], ref, f"config1 layer {l}, single")
 
 
 def test_config3_layer(salt_lib, oracle_mod, wl):

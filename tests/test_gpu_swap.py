@@ -118,3 +118,31 @@ def test_blob_checks(salt_lib, wl):
         with pytest.raises(salt.SaltError) as e:
             salt.salt_residual_load(r.ctx, 8, good, None)
         assert e.value.name == "SALT_ERR_SLOT_RANGE"
+
+
+def test_huge_page_host_blob_swap(salt_lib, oracle_mod, wl):
+    # salt_host_alloc memory is page-locked: a blob packed into it swaps in
+    # asynchronously and the apply reads the new residual.
+    from paper_2608_03579_gb300.runner import SaltRunner, bf16_bits, bf16_tensor
+    salt = salt_lib
+    w = _workload(wl)
+    with SaltRunner(w) as r:
+        r.pin_centroids()
+        r.load_slots()
+        nb = r.blob_bytes(2)
+        hb = salt.salt_host_alloc(3 * nb + 1000)
+        try:
+            assert hb.nbytes == 3 * nb + 1000 and int(hb.tensor[:4096].sum()) == 0
+            blob = hb.tensor[nb:2 * nb]
+            r.make_blob(2, version=5, out=blob)
+            side = torch.cuda.Stream()
+            salt.salt_residual_load(r.ctx, 2, blob, side)
+            r.build()
+            x = bf16_tensor(w.x(0))
+            y = bf16_tensor(w.y_in(0))
+            salt.salt_lora_apply(r.ctx, r.seg, 0, x, y)
+            torch.cuda.synchronize()
+            got = bf16_bits(y)
+        finally:
+            hb.close()
+    assert_close(got, _oracle(oracle_mod, w, lambda u: 5 if u == 2 else 0), "huge-page host blob")
