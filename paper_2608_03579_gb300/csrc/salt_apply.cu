@@ -26,8 +26,8 @@
 //       as bf16.  Each unit then counts its rows as written.
 //   expand items (row block, 64 output columns), cost-balanced over CTAs:
 //       Y[M x 64] += V_ext * Stack_B[:, cols] on the tensor cores (V_ext
-//       K-major, the B rows MN-major as they lie in memory, fp32 accumulators
-//       double-buffered in tensor memory), the y and B rows of the next items
+//       K-major, the B rows MN-major as they lie in memory, four fp32
+//       accumulators in tensor memory), the y and B rows of the next items
 //       streaming through the ring meanwhile.  A run of items of one block
 //       starts by prefetching its first items, then waits (bounded) until
 //       every row of the block's V tile is written.  y is read once and
@@ -60,7 +60,8 @@ constexpr int PRODUCER_WARPS = 3;              // expand roles: producers, one M
 constexpr int PRODUCER_THREADS = 32 * PRODUCER_WARPS;
 constexpr int EPI_WARPS = 4;
 static_assert(PRODUCER_WARPS + 1 + EPI_WARPS == APPLY_THREADS / 32, "expand warp roles cover the CTA");
-constexpr int TMEM_COLS = 128;                 // shrink: D^T (<= 128 tokens); expand: 2 x 64 columns
+constexpr int TMEM_COLS = 256;                 // shrink: D^T (<= 128 tokens); expand: N_ACC x 64 columns
+constexpr int N_ACC = 4;                       // expand accumulators in tensor memory
 constexpr int KS_MAX = 16;
 constexpr int VT_ROW = VEXT_COLS * 2;          // bytes per V tile row
 constexpr int VT_BYTES = TM * VT_ROW;
@@ -78,7 +79,7 @@ struct FusedInfo {
     int16_t rt1[S_MAX];          //                    -> one past the last token
     int16_t rk[S_MAX];           //                    -> rank index within the user
     uint64_t bar[A_MAX_STAGES];  // shrink: per stage, its MMAs have completed
-    uint64_t bbar[2 * B_MAX_STAGES + 5];  // expand: full, empty per stage; acc full, acc empty; V full
+    uint64_t bbar[2 * B_MAX_STAGES + 2 * N_ACC + 1];  // expand: full, empty per stage; acc full, acc empty; V full
     int32_t range[4];            // expand: first item (block, unit), end item (block, unit)
     uint32_t tmem;
     uint32_t epoch;
@@ -118,9 +119,13 @@ __device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar)
 {
     asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(bar) : "memory");
 }
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+// Relaxed arrive: orders nothing by itself, so it does not wait for this
+// thread's global stores.  Used where what the barrier guards is already
+// ordered: shared-memory values consumed into registers before the arrive,
+// tensor-memory loads completed by tcgen05.wait::ld.
+__device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar)
 {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+    asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
 }
 // barrier among the first n threads of the CTA (n a multiple of 32), id 1..15
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory"); }
@@ -562,7 +567,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     //   warps 0-2  producers: cp.async of each item's y rows and stacked B
     //              rows into a stage; each thread's copies complete on the
     //              stage's "full" barrier; the V tile once per run;
-    //   warp 3     one thread issues the MMAs of an item into one of two
+    //   warp 3     one thread issues the MMAs of an item into one of N_ACC
     //              accumulators and commits them to "acc full" and "empty";
     //   warps 4-7  epilogue: TMEM lanes 32 (w % 4) .. + 31 (one token row a
     //              thread), the item's 64 columns: + staged y, one rounding,
@@ -576,17 +581,17 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     auto full_bar = [&](int st) { return bb + 8u * st; };
     auto empty_bar = [&](int st) { return bb + 8u * (B_MAX_STAGES + st); };
     auto accf_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + i); };
-    auto acce_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + 2 + i); };
-    const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 4);
+    auto acce_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + N_ACC + i); };
+    const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 2 * N_ACC);
     // The barriers are set up once; their phases run on across runs: item g
     // (counted over all runs of this CTA) uses slot g % B_MAX_STAGES and
-    // accumulator g & 1, the r-th run's V tile the r-th phase of "V full".
+    // accumulator g % N_ACC, the r-th run's V tile the r-th phase of "V full".
     if (tid == 0) {
         for (int st = 0; st < B_MAX_STAGES; ++st) {
             mbar_init(full_bar(st), PRODUCER_THREADS);
             mbar_init(empty_bar(st), 1 + EPI_WARPS);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < N_ACC; ++i) {
             mbar_init(accf_bar(i), 1);
             mbar_init(acce_bar(i), EPI_WARPS);
         }
@@ -679,9 +684,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             if (lane == 0) {
                 if (!mbar_wait(vfull_bar, runs & 1)) ok_all = false;
                 for (int j = 0; j < n; ++j) {
-                    const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g & 1;
+                    const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g % N_ACC;
                     if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
-                    if (g >= 2 && !mbar_wait(acce_bar(buf), ((g >> 1) - 1) & 1)) ok_all = false;
+                    if (g >= N_ACC && !mbar_wait(acce_bar(buf), ((g / N_ACC) - 1) & 1)) ok_all = false;
                     fence_async_smem();
                     tc_fence_after();
                     const uint32_t sb = ring32 + (j % nbs) * bst + m_rows * 128;
@@ -697,9 +702,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             const int q = warp & 3;
             const int row = q * 32 + lane;
             for (int j = 0; j < n; ++j) {
-                const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g & 1;
+                const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g % N_ACC;
                 const int st = j % nbs;
-                if (!mbar_wait(accf_bar(buf), (g >> 1) & 1)) ok_all = false;
+                if (!mbar_wait(accf_bar(buf), (g / N_ACC) & 1)) ok_all = false;
                 tc_fence_after();
                 uint32_t acc[64];
                 const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + buf * NC;
@@ -708,7 +713,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 tmem_ld_wait();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(acce_bar(buf));
+                if (lane == 0) mbar_arrive_relaxed(acce_bar(buf));
                 // the staged y rows of the item (its "full" phase has completed)
                 if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
                 // y + delta, rounded once, back into the staged tile (this
@@ -737,16 +742,23 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 }
                 __syncwarp();
                 // ... then the warp's 32 rows go out whole: 8 lanes per
-                // 128-byte row piece, 4 rows per store
+                // 128-byte row piece, 4 rows per store (all reads first)
+                {
+                    uint4 vv[8];
+                    int64_t off[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = q * 32 + i * 4 + (lane >> 3), c = lane & 7, col = n0 + c * 8;
-                    if (r < M && col < d_out)
-                        *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.row[r] * d_out + col) =
-                            *reinterpret_cast<const uint4 *>(ysp + swz128(r, c));
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = q * 32 + i * 4 + (lane >> 3), c = lane & 7, col = n0 + c * 8;
+                        const bool ok = r < M && col < d_out;
+                        vv[i] = ok ? *reinterpret_cast<const uint4 *>(ysp + swz128(r, c)) : make_uint4(0u, 0u, 0u, 0u);
+                        off[i] = ok ? (int64_t)info.row[r] * d_out + col : -1;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        if (off[i] >= 0) *reinterpret_cast<uint4 *>(pr.y + off[i]) = vv[i];
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(empty_bar(slot));
+                if (lane == 0) mbar_arrive_relaxed(empty_bar(slot));
             }
         }
         g0 += n;
