@@ -1,6 +1,6 @@
 """Shared helpers of the GPU parity tests: oracle tables and the tolerance.
 
-Tolerance (the benchmark spec, bf16 inputs with fp32 accumulation):
+Tolerance of the serving path (bf16 inputs with fp32 accumulation):
 |y_gpu - y_ref| <= 2e-2 * |y_ref| + 2e-2 * max|y_ref|, the max taken over the
 output tensor of the call (or of the sampled rows).  Index outputs are
 compared bit for bit.
