@@ -127,8 +127,24 @@ __device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar)
 {
     asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
 }
+// arrive on the mbarrier, adding `bytes` to the transaction count its phase waits for
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+}
+// 2-D TMA tile load (coordinates in elements, x first) completing on bar by bytes
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+        "l"(map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
 // barrier among the first n threads of the CTA (n a multiple of 32), id 1..15
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory"); }
+// order global data this thread observed through the generic proxy before
+// async-proxy (TMA) reads of it
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;\n" ::: "memory"); }
 
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
@@ -595,7 +611,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             mbar_init(accf_bar(i), 1);
             mbar_init(acce_bar(i), EPI_WARPS);
         }
-        mbar_init(vfull_bar, PRODUCER_THREADS);
+        mbar_init(vfull_bar, 1);
         mbar_fence_init();
     }
     __syncthreads();
@@ -654,25 +670,23 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 cp_async_commit();
                 cp_async_arrive_noinc(full_bar((g0 + j) % B_MAX_STAGES));
             };
-            const int npre = min(n, nbs);
-            for (int j = 0; j < npre; ++j) load_item(j);
-            // V: once every row of the block's tile is written
+            // V first: once every row of the block's tile is written, two TMA
+            // tile loads (K 0..63 and 64..127, each straight into the K-major
+            // 128-byte-swizzled layout) complete on "V full" by byte count.
+            // Issued before the item copies, it does not wait behind them.
             if (tid == 0) {
                 const int n_ne = min(KS, (pr.d_in + KC - 1) / KC);
                 if (!wait_count(p.w.vdone + (epoch & 1) * n_pairs + ((int64_t)pi * p.w.blk_cap + cb), n_ne))
                     ok_all = false;
+                fence_proxy_async_global();  // the tile was written through the generic proxy
+                const int row0 = (int)(((int64_t)pi * p.w.blk_cap + cb) * TM);
+                mbar_expect_tx(vfull_bar, 2 * TILE_BYTES);
+                tma_load_2d(vs32, &p.w.vmap, 0, row0, vfull_bar);
+                tma_load_2d(vs32 + TILE_BYTES, &p.w.vmap, 64, row0, vfull_bar);
             }
-            named_sync(1, PRODUCER_THREADS);
-            {
-                const uint16_t *vt = p.w.vext + ((int64_t)pi * p.w.blk_cap + cb) * (TM * VEXT_COLS);
-                const int nch = S_pad >> 3;
-                for (int idx = tid; idx < M * nch; idx += PRODUCER_THREADS) {
-                    const int r = idx / nch, c = idx - r * nch;
-                    cp_async16(vs32 + (c >> 3) * TILE_BYTES + swz128(r, c & 7), vt + (int64_t)r * VEXT_COLS + c * 8, true);
-                }
-                cp_async_commit();
-                cp_async_arrive_noinc(vfull_bar);
-            }
+            named_sync(1, PRODUCER_THREADS);  // the item copies go out after V
+            const int npre = min(n, nbs);
+            for (int j = 0; j < npre; ++j) load_item(j);
             for (int j = npre; j < n; ++j) {
                 // the stage last held item j - nbs of this run
                 const uint32_t gp = g0 + j - nbs;
@@ -823,10 +837,38 @@ cudaError_t apply_static_workspace(ApplyWork *out)
         w.arrive = static_cast<uint32_t *>(c);
         w.vdone = static_cast<uint32_t *>(d);
         w.seq = static_cast<uint32_t *>(f);
+        if ((e = apply_encode_vmap(w)) != cudaSuccess) return e;
         ws[dev] = w;
     }
     *out = ws[dev];
     return cudaSuccess;
+}
+
+cudaError_t apply_encode_vmap(ApplyWork &w)
+{
+    using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+    static Encode encode = nullptr;
+    static std::mutex mu;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (!encode) {
+            void *fn = nullptr;
+            cudaDriverEntryPointQueryResult q;
+            cudaError_t e = cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &fn, cudaEnableDefault, &q);
+            if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return e != cudaSuccess ? e : cudaErrorNotSupported;
+            encode = reinterpret_cast<Encode>(fn);
+        }
+    }
+    const cuuint64_t dims[2] = {(cuuint64_t)VEXT_COLS, (cuuint64_t)SALT_MAX_GROUP * w.blk_cap * TM};
+    const cuuint64_t strides[1] = {(cuuint64_t)VEXT_COLS * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)TM};
+    const cuuint32_t es[2] = {1, 1};
+    const CUresult r = encode(&w.vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.vext, dims, strides, box, es,
+                              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
 cudaError_t apply_prepare(int device)

@@ -2,6 +2,7 @@
 // kernels (salt_segments.cu, salt_apply.cu).  Not part of the public ABI.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -30,9 +31,9 @@ constexpr int BLK_START = 0, BLK_LEN = 1, BLK_DOM = 2, BLK_RC = 3, BLK_NRES = 4,
 
 // Cost of one 64-column expand item of a block in 128-byte rows moved: y
 // read and written (2 M), the stacked B rows (S), plus a fixed share for the
-// per-item handoffs between the expand's warp roles (measured at about
-// 0.5 us an item, 128 rows' worth at the per-SM streaming rate).
-__host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 128; }
+// per-item handoffs between the expand's warp roles (an item was measured to
+// take about 1 us whatever its size, so the fixed share dominates).
+__host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 384; }
 
 // Device arrays of one segments object.
 struct SegDev {
@@ -69,6 +70,9 @@ struct SegDev {
 //   seq:    [0] launch counter (the epoch), [1] CTAs of the running launch
 //           that have finished.
 struct ApplyWork {
+    // TMA map of vext as a 2-D bf16 tensor [rows][VEXT_COLS], box 64 x TM,
+    // 128-byte swizzle (the K-major UMMA layout of a V tile half)
+    alignas(64) CUtensorMap vmap;
     uint16_t *vext;        // [SALT_MAX_GROUP * blk_cap * TM * VEXT_COLS]
     int32_t blk_cap;
     float *part;           // [part_cap * TM * PART_COLS]
@@ -123,6 +127,9 @@ struct ApplyParams {
     ApplyWork w;
     uint32_t *err;
 };
+
+// Encode w.vmap for w.vext and w.blk_cap (host; once per workspace).
+cudaError_t apply_encode_vmap(ApplyWork &w);
 
 // Kernel launchers (defined next to the kernels).
 cudaError_t launch_segments(const SegParams &p, cudaStream_t stream);

@@ -537,7 +537,8 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
          cudaMalloc(&seg->work.seq, 2 * sizeof(uint32_t)) == cudaSuccess &&
          cudaMemset(seg->work.arrive, 0, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
          cudaMemset(seg->work.vdone, 0, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
-         cudaMemset(seg->work.seq, 0, 2 * sizeof(uint32_t)) == cudaSuccess;
+         cudaMemset(seg->work.seq, 0, 2 * sizeof(uint32_t)) == cudaSuccess &&
+         apply_encode_vmap(seg->work) == cudaSuccess;
     for (int i = 0; ok && i < 2; ++i) {
         ok = cudaHostAlloc(&seg->staging[i], 2 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
              cudaEventCreateWithFlags(&seg->staging_ev[i], cudaEventDisableTiming) == cudaSuccess;
