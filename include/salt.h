@@ -306,6 +306,18 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg, int3
                                    const void *x, void *y, salt_stream_t stream);
 
 /*
+ * Self-test of the failure path.  Enqueues on `stream` one thread that
+ * waits, with the same bounded wait the apply uses for results of other
+ * CTAs (the V rows of a row block), on a device word nothing ever sets.  The
+ * wait gives up after its limit (a fraction of a second), raises
+ * SALT_DEVERR_TIMEOUT in the device error word and returns; the context and
+ * the GPU stay usable.  Read the flag with salt_get_device_error.  (The
+ * paper has no counterpart; it demonstrates that a lost result produces an
+ * error status instead of a hang.)
+ */
+salt_status salt_selftest_wait_timeout(salt_ctx *ctx, salt_stream_t stream);
+
+/*
  * Synchronise `stream`, then read and clear the device error word.
  * *flags gets the SALT_DEVERR_* bits raised since the last call.  Returns
  * SALT_ERR_DEVICE_IDS if any bit was set, else SALT_OK.

@@ -807,6 +807,16 @@ __device__ __align__(256) uint32_t g_static_seq[2];
 // SM count per device (the grid of the apply kernel), filled by apply_prepare
 int g_sm_count[64];
 
+// A device word nothing ever writes: the failure-path self-test waits on it.
+__device__ uint32_t g_never_set;
+
+// One thread waits for g_never_set to read 1 through the bounded wait the
+// apply uses for other CTAs' results; it gives up and raises the timeout flag.
+__global__ void salt_wait_selftest_kernel(uint32_t *err)
+{
+    if (threadIdx.x == 0 && blockIdx.x == 0 && !wait_count(&g_never_set, 1u)) atomicOr(err, SALT_DEVERR_TIMEOUT);
+}
+
 }  // namespace
 
 size_t apply_smem_bytes() { return FUSED_SMEM; }
@@ -877,6 +887,12 @@ cudaError_t apply_prepare(int device)
     cudaError_t e = cudaDeviceGetAttribute(&g_sm_count[device], cudaDevAttrMultiProcessorCount, device);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(salt_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FUSED_SMEM);
+}
+
+cudaError_t launch_wait_selftest(uint32_t *err, cudaStream_t stream)
+{
+    salt_wait_selftest_kernel<<<1, 32, 0, stream>>>(err);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_apply(const ApplyParams &p, bool pdl, cudaStream_t stream)

@@ -140,6 +140,9 @@ cudaError_t apply_prepare(int device);
 // the stream (only when that kernel did not write the segment tables).
 cudaError_t launch_apply(const ApplyParams &p, bool pdl, cudaStream_t stream);
 size_t apply_smem_bytes();
+// One thread waits, with the apply's bounded cross-CTA wait, on a device word
+// nothing sets; raises SALT_DEVERR_TIMEOUT in *err when it gives up.
+cudaError_t launch_wait_selftest(uint32_t *err, cudaStream_t stream);
 
 // Row blocks and partial tiles the allocation-free apply
 // (salt_lora_apply_static) can use from its static device scratch.

@@ -840,6 +840,14 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     return SALT_OK;
 }
 
+salt_status salt_selftest_wait_timeout(salt_ctx *ctx, salt_stream_t stream)
+{
+    if (!ctx) return SALT_ERR_INVALID_ARG;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, launch_wait_selftest(ctx->err_dev, static_cast<cudaStream_t>(stream)));
+    return SALT_OK;
+}
+
 salt_status salt_get_device_error(salt_ctx *ctx, salt_stream_t stream, uint32_t *flags)
 {
     if (!ctx || !flags) return SALT_ERR_INVALID_ARG;

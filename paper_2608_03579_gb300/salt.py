@@ -76,6 +76,7 @@ _SIGS = {
     "salt_lora_apply_grouped": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
     "salt_lora_apply_static": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp]),
     "salt_get_device_error": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]),
+    "salt_selftest_wait_timeout": (ctypes.c_int, [_vp, _vp]),
     "salt_host_alloc": (_vp, [_i64]),
     "salt_host_free": (None, [_vp]),
 }
@@ -259,6 +260,10 @@ def salt_lora_apply_grouped(ctx, seg, layers, xs, ys, stream=None) -> None:
     xa = (ctypes.c_void_p * n)(*[_ptr(t) for t in xs])
     ya = (ctypes.c_void_p * n)(*[_ptr(t) for t in ys])
     _check(_lib.salt_lora_apply_grouped(ctx, seg, n, la, xa, ya, _stream(stream)), ctx)
+
+
+def salt_selftest_wait_timeout(ctx, stream=None) -> None:
+    _check(_lib.salt_selftest_wait_timeout(ctx, _stream(stream)), ctx)
 
 
 def salt_get_device_error(ctx, stream=None, raise_on_flags: bool = False) -> int:
