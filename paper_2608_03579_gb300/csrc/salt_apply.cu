@@ -53,10 +53,10 @@ namespace {
 constexpr int KC = 64;                         // K chunk of the shrink (128-byte rows)
 constexpr int NC = 64;                         // output columns per expand item
 constexpr int TILE_BYTES = TM * 128;           // 128 rows x 128 B
-constexpr int RING_BYTES = 192 * 1024;         // shared-memory ring of both phases
+constexpr int RING_BYTES = 216 * 1024;         // shared-memory ring of both phases
 constexpr int A_MAX_STAGES = 8;
 constexpr int B_MAX_STAGES = 10;               // expand: stages of (y rows | stacked B rows) per item
-constexpr int PRODUCER_WARPS = 3;              // expand roles: producers, one MMA warp, epilogue warps
+constexpr int PRODUCER_WARPS = 7;              // expand roles: producers, one MMA warp, epilogue warps
 constexpr int PRODUCER_THREADS = 32 * PRODUCER_WARPS;
 constexpr int EPI_WARPS = 4;
 static_assert(PRODUCER_WARPS + 1 + EPI_WARPS == APPLY_THREADS / 32, "expand warp roles cover the CTA");
@@ -449,7 +449,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         tc_fence_after();
 
         // ---- D^T (TMEM lanes = stack rows, columns = tokens).  Warp w reads
-        // lanes 32 (w % 4) .. + 31 and every other 16-token group.
+        // lanes 32 (w % 4) .. + 31 and every (warps / 4)-th 16-token group.
         const int q = warp & 3, th = warp >> 2;
         const int sr = q * 32 + lane;
         int t0 = 0, t1 = 0, col = -1;  // tokens this stack row serves, its compact column
@@ -468,7 +468,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         const int nch = S_pad >> 3;
         if (KS == 1) {
             // V_ext straight from the accumulator into the staging tile
-            for (int g = th; g < (m_rows >> 4); g += 2) {
+            for (int g = th; g < (m_rows >> 4); g += APPLY_THREADS / 128) {
                 uint32_t v[16];
                 tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
                 tmem_ld_wait();
@@ -495,7 +495,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         } else {
             // fp32 partial: token t's centroid columns, then its own user's columns
             float *P = p.w.part + (int64_t)unit * (TM * PART_COLS);
-            for (int g = th; g < (m_rows >> 4); g += 2) {
+            for (int g = th; g < (m_rows >> 4); g += APPLY_THREADS / 128) {
                 uint32_t v[16];
                 tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
                 tmem_ld_wait();
@@ -580,12 +580,12 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
 
     // ================================================================ expand items
     // Warp roles per run of items of one (block, projection):
-    //   warps 0-2  producers: cp.async of each item's y rows and stacked B
+    //   warps 0-6  producers: cp.async of each item's y rows and stacked B
     //              rows into a stage; each thread's copies complete on the
     //              stage's "full" barrier; the V tile once per run;
-    //   warp 3     one thread issues the MMAs of an item into one of N_ACC
+    //   warp 7     one thread issues the MMAs of an item into one of N_ACC
     //              accumulators and commits them to "acc full" and "empty";
-    //   warps 4-7  epilogue: TMEM lanes 32 (w % 4) .. + 31 (one token row a
+    //   warps 8-11 epilogue: TMEM lanes 32 (w % 4) .. + 31 (one token row a
     //              thread), the item's 64 columns: + staged y, one rounding,
     //              store; then "acc empty" and "empty".
     int b = info.range[0], u = info.range[1];

@@ -16,7 +16,7 @@ namespace salt {
 // rows: rc_max + umax * r_max <= S_MAX.
 constexpr int TM = 128;
 constexpr int S_MAX = 128;
-constexpr int APPLY_THREADS = 256;
+constexpr int APPLY_THREADS = 384;  // 12 warps: in the expand 7 producers, 1 MMA, 4 epilogue
 constexpr int SEG_THREADS = 1024;
 
 constexpr int VEXT_COLS = S_MAX;    // row pitch (elements) of a block's V tile in the workspace
