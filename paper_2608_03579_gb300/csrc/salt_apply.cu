@@ -247,6 +247,7 @@ __device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, in
 }
 
 constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
+constexpr int N_QUADS = APPLY_THREADS / 128;  // full groups of 4 warps (one per TMEM lane quarter)
 
 __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __grid_constant__ ApplyParams p)
 {
@@ -448,8 +449,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             }
         tc_fence_after();
 
-        // ---- D^T (TMEM lanes = stack rows, columns = tokens).  Warp w reads
-        // lanes 32 (w % 4) .. + 31 and every (warps / 4)-th 16-token group.
+        // ---- D^T (TMEM lanes = stack rows, columns = tokens).  Warp w of the
+        // first N_QUADS groups of four reads lanes 32 (w % 4) .. + 31 and every
+        // N_QUADS-th 16-token group.
         const int q = warp & 3, th = warp >> 2;
         const int sr = q * 32 + lane;
         int t0 = 0, t1 = 0, col = -1;  // tokens this stack row serves, its compact column
@@ -468,7 +470,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         const int nch = S_pad >> 3;
         if (KS == 1) {
             // V_ext straight from the accumulator into the staging tile
-            for (int g = th; g < (m_rows >> 4); g += APPLY_THREADS / 128) {
+            for (int g = th; th < N_QUADS && g < (m_rows >> 4); g += N_QUADS) {
                 uint32_t v[16];
                 tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
                 tmem_ld_wait();
@@ -495,7 +497,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         } else {
             // fp32 partial: token t's centroid columns, then its own user's columns
             float *P = p.w.part + (int64_t)unit * (TM * PART_COLS);
-            for (int g = th; g < (m_rows >> 4); g += APPLY_THREADS / 128) {
+            for (int g = th; th < N_QUADS && g < (m_rows >> 4); g += N_QUADS) {
                 uint32_t v[16];
                 tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
                 tmem_ld_wait();
