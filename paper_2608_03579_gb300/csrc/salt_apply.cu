@@ -201,7 +201,8 @@ __device__ __forceinline__ const uint16_t *residual_row(const ApplyParams &p, co
 }
 
 // K-split s of KS over nk chunks: [nk * s / KS, nk * (s + 1) / KS)
-__device__ __forceinline__ int split_lo(int nk, int s, int KS) { return (int)((int64_t)nk * s / KS); }
+// (s <= KS <= 16, so nk * s fits 32 bits for any d_in below 8e9)
+__device__ __forceinline__ int split_lo(int nk, int s, int KS) { return nk * s / KS; }
 
 __device__ __forceinline__ int64_t blk_wend(const int32_t *blk, int b) { return blk[(int64_t)BLK_INTS * b + BLK_WEND]; }
 
@@ -519,9 +520,13 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 if (!wait_count(ctr, n_ne)) ok_all = false;
             }
             __syncthreads();
-            uint32_t ne_mask = 0;  // the non-empty splits
-            for (int s2 = 0; s2 < KS; ++s2)
-                if (nk >= KS || split_lo(nk, s2 + 1, KS) > split_lo(nk, s2, KS)) ne_mask |= 1u << s2;
+            // the non-empty splits: all of them unless d_in has fewer chunks than splits
+            uint32_t ne_mask = KS >= 32 ? ~0u : (1u << KS) - 1u;
+            if (nk < KS) {
+                ne_mask = 0;
+                for (int s2 = 0; s2 < KS; ++s2)
+                    if (split_lo(nk, s2 + 1, KS) > split_lo(nk, s2, KS)) ne_mask |= 1u << s2;
+            }
             const int si = nk >= KS ? s : c0;  // index among the non-empty splits
             const int r0 = M * si / n_ne, r1 = M * (si + 1) / n_ne;
             float *Ps = reinterpret_cast<float *>(ring);  // [r1 - r0][PART_COLS] sums
