@@ -275,15 +275,6 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     const int n_units = n_bp * KS;
     const int ua = (int)((int64_t)n_units * blockIdx.x / gridDim.x);
     const int ub = (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
-    const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
-    if (warp < 2) {
-        int b, u;
-        item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + warp) / gridDim.x, lane, b, u);
-        if (lane == 0) {
-            info.range[2 * warp] = b;
-            info.range[2 * warp + 1] = u;
-        }
-    }
     if (warp == 2) {
         tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
         tmem_relinquish();
@@ -312,6 +303,21 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         for (int i = blockIdx.x * APPLY_THREADS + tid; i < n_pairs; i += gridDim.x * APPLY_THREADS) {
             p.w.arrive[nxt + i] = 0u;
             p.w.vdone[nxt + i] = 0u;
+        }
+    };
+
+    // This CTA's share of the expand items: the first (e = 0) or end (e = 1)
+    // item of its cost range, into info.range; one warp each.  Searched while
+    // the CTA waits for the other splits of its block (or at the end of the
+    // shrink phase): its dependent reads would otherwise delay the start.
+    bool have_range = false;
+    auto find_range = [&](int e) {
+        const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
+        int b, u;
+        item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + e) / gridDim.x, lane, b, u);
+        if (lane == 0) {
+            info.range[2 * e] = b;
+            info.range[2 * e + 1] = u;
         }
     };
 
@@ -518,7 +524,10 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 uint32_t *ctr = p.w.arrive + (info.epoch & 1) * n_pairs + pidx;
                 signal_add(ctr);
                 if (!wait_count(ctr, n_ne)) ok_all = false;
+            } else if (!have_range && (warp == 1 || warp == 2)) {
+                find_range(warp - 1);  // meanwhile: this CTA's share of the expand items
             }
+            have_range = true;
             __syncthreads();
             // the non-empty splits: all of them unless d_in has fewer chunks than splits
             uint32_t ne_mask = KS >= 32 ? ~0u : (1u << KS) - 1u;
@@ -580,6 +589,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         if (tid == 0) signal_add(p.w.vdone + (info.epoch & 1) * n_pairs + pidx);
     }
     if (!waited) dep_wait();
+    if (!have_range && warp < 2) find_range(warp);
     tc_fence_before();
     __syncthreads();  // the shrink phase is over: ring and tensor memory change hands
     tc_fence_after();
