@@ -292,18 +292,12 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     // its outputs), then read this launch's epoch; its parity selects the
     // half of the counters this launch uses.
     const int n_pairs = SALT_MAX_GROUP * p.w.blk_cap;
+    // (No barrier here: the epoch is first used after the K loop, whose CTA
+    // barriers publish it; the x loads need not wait for it.)
     auto dep_wait = [&]() {
         pdl_wait();
         waited = true;
         if (tid == 0) info.epoch = *reinterpret_cast<volatile uint32_t *>(p.w.seq);
-        __syncthreads();
-        // the counters of the next launch start from zero (the previous
-        // launch, which used them, is complete)
-        const int nxt = ((info.epoch + 1) & 1) * n_pairs;
-        for (int i = blockIdx.x * APPLY_THREADS + tid; i < n_pairs; i += gridDim.x * APPLY_THREADS) {
-            p.w.arrive[nxt + i] = 0u;
-            p.w.vdone[nxt + i] = 0u;
-        }
     };
 
     // This CTA's share of the expand items: the first (e = 0) or end (e = 1)
@@ -594,6 +588,15 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     __syncthreads();  // the shrink phase is over: ring and tensor memory change hands
     tc_fence_after();
     const uint32_t epoch = info.epoch;
+    // the counters of the next launch start from zero (the previous launch,
+    // which used them, is complete)
+    {
+        const int nxt = ((epoch + 1) & 1) * n_pairs;
+        for (int i = blockIdx.x * APPLY_THREADS + tid; i < n_pairs; i += gridDim.x * APPLY_THREADS) {
+            p.w.arrive[nxt + i] = 0u;
+            p.w.vdone[nxt + i] = 0u;
+        }
+    }
 
     // ================================================================ expand items
     // Warp roles per run of items of one (block, projection):
