@@ -498,10 +498,12 @@ def run_salt(args, rank, world, local, pg):
     # e2e: host buffers, copies inside the timed region
     e2e = None
     if not args.no_e2e:
-        x_host = torch.empty(st.x_elems, dtype=torch.bfloat16, pin_memory=True)
+        # host activations in huge-page page-locked memory (salt_host_alloc):
+        # ordinary pinned pages stall the copy engine under sustained transfers
+        hb = [st.salt.salt_host_alloc(n * 2) for n in (st.x_elems, st.y_elems, st.y_elems)]
+        x_host, y_host, y_out = (h.tensor.view(torch.bfloat16) for h in hb)
         x_host.copy_(st.x_all)
-        y_host = torch.zeros(st.y_elems, dtype=torch.bfloat16, pin_memory=True)
-        y_out = torch.empty(st.y_elems, dtype=torch.bfloat16, pin_memory=True)
+        y_host.zero_()
         torch.cuda.synchronize(local)
         n_e2e = max(3, min(args.steps, 10))
         barrier(pg, local)
@@ -522,6 +524,9 @@ def run_salt(args, rank, world, local, pg):
         h2d = st.x_elems * 2 + st.y_elems * 2 + 2 * st.T * 4 + st.wl_mod.C4_REGION * st.blob_bytes
         e2e = {"value": world * st.T / (e2e_ms / 1000.0), "unit": "tokens/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(st.y_elems * 2)}
+        x_host = y_host = y_out = None
+        for h in hb:
+            h.close()
 
     # swap-only and apply-only reference timings (context for the step time)
     swap_ms = None
