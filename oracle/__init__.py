@@ -8,9 +8,11 @@ package: the two share no code.  The arithmetic lives in ``salt_oracle.c``
 compiler and marshals numpy arrays through ctypes.
 
 Paper sections followed: "Multi-Tenant Serving" (W_final = W_base +
-gamma*Wbar + delta_i, the grouping of requests by centroid), "The
+gamma*Wbar + delta_i, the grouping of requests by their (centroid, gamma)
+pair, the fold of a scaled centroid into the base weights), "The
 Centroid-Residual Decomposition" (Wbar and delta_i as low-rank products),
-and the memory columns of Table 1 and the appendix tables (adapter bytes).
+Eq. 2 (the alignment regulariser of Phase 1) and the memory columns of
+Table 1 and the appendix tables (adapter bytes).
 """
 from __future__ import annotations
 
@@ -35,7 +37,7 @@ def build(force: bool = False) -> str:
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-ffp-contract=off",
-           "-o", tmp, _SRC]
+           "-o", tmp, _SRC, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
@@ -45,12 +47,17 @@ def _configure(lib):
     vp = ctypes.c_void_p
     i32, i64 = ctypes.c_int32, ctypes.c_int64
     lib.oracle_apply.restype = ctypes.c_int
-    lib.oracle_apply.argtypes = [i64, i64, i64, vp, vp, vp, vp,
+    lib.oracle_apply.argtypes = [i64, i64, i64, vp, vp, vp, vp, vp,
                                  i32, vp, vp, vp, vp,
                                  i32, vp, vp, vp, vp,
                                  i64, vp, vp]
     lib.oracle_segments.restype = ctypes.c_int
-    lib.oracle_segments.argtypes = [i32, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.oracle_segments.argtypes = [i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+    f64 = ctypes.c_double
+    lib.oracle_align_loss.restype = ctypes.c_int
+    lib.oracle_align_loss.argtypes = [i64, i64, i32, vp, vp, f64, i32, vp, vp, f64, f64, vp]
+    lib.oracle_fold.restype = ctypes.c_int
+    lib.oracle_fold.argtypes = [i64, i64, i32, vp, vp, f64, vp, i32, vp]
     lib.oracle_adapter_bytes.restype = i64
     lib.oracle_adapter_bytes.argtypes = [i32, vp, vp, i32]
     return lib
@@ -85,11 +92,12 @@ def _ptr_array(arrs):
     return out, keep
 
 
-def apply(x, y_in, dom, slot, centroids, residuals, rows=None):
+def apply(x, y_in, dom, slot, centroids, residuals, rows=None, gamma=None):
     """Evaluate one projection for the listed tokens in fp64.
 
     x: uint16 [T, d_in] (bf16 bits); y_in: uint16 [T, d_out] or None.
     dom, slot: int32 [T], -1 drops the term.
+    gamma: float64 [T] factor on each token's centroid term, or None (1).
     centroids: list over domains of (At [rc, d_in] uint16, B [rc, d_out] uint16, s_c)
                or None for an absent domain.
     residuals: list over slots of (At [r, d_in], B [r, d_out], s_u) or None.
@@ -143,8 +151,12 @@ def apply(x, y_in, dom, slot, centroids, residuals, rows=None):
         rows_arr = np.ascontiguousarray(rows, dtype=np.int64)
         n_rows = rows_arr.shape[0]
     out = np.zeros((n_rows, d_out), dtype=np.float64)
+    if gamma is not None:
+        gamma = np.ascontiguousarray(gamma, dtype=np.float64)
+        if gamma.shape != (T,):
+            raise ValueError("gamma must hold one factor per token")
     rc_ = lib.oracle_apply(T, d_in, d_out, _ptr(x), _ptr(y_in) if y_in is not None else None,
-                           _ptr(dom), _ptr(slot),
+                           _ptr(dom), _ptr(slot), _ptr(gamma) if gamma is not None else None,
                            nd, _ptr(rc), _ptr(s_c), pAc, pBc,
                            ns, _ptr(ru), _ptr(s_u), pAu, pBu,
                            n_rows, _ptr(rows_arr) if rows_arr is not None else None, _ptr(out))
@@ -154,25 +166,31 @@ def apply(x, y_in, dom, slot, centroids, residuals, rows=None):
     return out
 
 
-def segments(dom, slot):
-    """Grouping oracle: stable sort by (domain, slot), then maximal runs.
+def segments(dom, slot, gbin=None):
+    """Grouping oracle: stable sort by (domain, gamma bin, slot), then
+    maximal runs.  gbin: int32 [T] gamma bins, or None (no bins).
 
-    Returns a dict of int32 arrays: perm, dseg_ptr, dseg_dom, useg_ptr,
-    useg_dom, useg_slot (each trimmed to its count).
+    Returns a dict of int32 arrays: perm, dseg_ptr, dseg_dom, dseg_gbin,
+    useg_ptr, useg_dom, useg_gbin, useg_slot (each trimmed to its count).
     """
     lib = _load()
     dom = np.ascontiguousarray(dom, dtype=np.int32)
     slot = np.ascontiguousarray(slot, dtype=np.int32)
+    if gbin is not None:
+        gbin = np.ascontiguousarray(gbin, dtype=np.int32)
     T = dom.shape[0]
     perm = np.zeros(max(1, T), dtype=np.int32)
     dptr = np.zeros(T + 1, dtype=np.int32)
     ddom = np.zeros(max(1, T), dtype=np.int32)
+    dgb = np.zeros(max(1, T), dtype=np.int32)
     uptr = np.zeros(T + 1, dtype=np.int32)
     udom = np.zeros(max(1, T), dtype=np.int32)
+    ugb = np.zeros(max(1, T), dtype=np.int32)
     uslot = np.zeros(max(1, T), dtype=np.int32)
     counts = np.zeros(2, dtype=np.int32)
-    rc = lib.oracle_segments(T, _ptr(dom), _ptr(slot), _ptr(perm), _ptr(dptr), _ptr(ddom),
-                             _ptr(uptr), _ptr(udom), _ptr(uslot), _ptr(counts))
+    rc = lib.oracle_segments(T, _ptr(dom), _ptr(gbin) if gbin is not None else None, _ptr(slot),
+                             _ptr(perm), _ptr(dptr), _ptr(ddom), _ptr(dgb),
+                             _ptr(uptr), _ptr(udom), _ptr(ugb), _ptr(uslot), _ptr(counts))
     if rc != 0:
         raise ValueError(f"oracle_segments failed with {rc}")
     nd, nu = int(counts[0]), int(counts[1])
@@ -180,10 +198,53 @@ def segments(dom, slot):
         "perm": perm[:T].copy(),
         "dseg_ptr": dptr[:nd + 1].copy(),
         "dseg_dom": ddom[:nd].copy(),
+        "dseg_gbin": dgb[:nd].copy(),
         "useg_ptr": uptr[:nu + 1].copy(),
         "useg_dom": udom[:nu].copy(),
+        "useg_gbin": ugb[:nu].copy(),
         "useg_slot": uslot[:nu].copy(),
     }
+
+
+def align_loss(At, B, s, At_c, B_c, s_c, eps=1e-8):
+    """Eq. 2 from the dense matrices Delta W = s*A B and Wbar = s_c*A_c B_c.
+
+    At [r, d_in], B [r, d_out], At_c [rc, d_in], B_c [rc, d_out]: uint16
+    bf16 bits.  Returns a dict: loss, cosine, trace, norm_dw, norm_wbar.
+    """
+    lib = _load()
+    At = np.ascontiguousarray(At, dtype=np.uint16)
+    B = np.ascontiguousarray(B, dtype=np.uint16)
+    At_c = np.ascontiguousarray(At_c, dtype=np.uint16)
+    B_c = np.ascontiguousarray(B_c, dtype=np.uint16)
+    r, d_in = At.shape
+    rc = At_c.shape[0]
+    d_out = B.shape[1] if r else B_c.shape[1]
+    if B.shape != (r, d_out) or At_c.shape != (rc, d_in) or B_c.shape != (rc, d_out):
+        raise ValueError("factor shapes do not match")
+    out = np.zeros(5, dtype=np.float64)
+    rc_ = lib.oracle_align_loss(d_in, d_out, r, _ptr(At), _ptr(B), float(s),
+                                rc, _ptr(At_c), _ptr(B_c), float(s_c), float(eps), _ptr(out))
+    if rc_ != 0:
+        raise ValueError(f"oracle_align_loss failed with {rc_}")
+    return {"loss": out[0], "cosine": out[1], "trace": out[2], "norm_dw": out[3], "norm_wbar": out[4]}
+
+
+def fold(At_c, B_c, scale, W, layout):
+    """W + scale * A_c B_c in fp64 (layout 0: W [d_in, d_out]; 1: W [d_out, d_in])."""
+    lib = _load()
+    At_c = np.ascontiguousarray(At_c, dtype=np.uint16)
+    B_c = np.ascontiguousarray(B_c, dtype=np.uint16)
+    W = np.ascontiguousarray(W, dtype=np.uint16)
+    rc, d_in = At_c.shape
+    d_out = B_c.shape[1]
+    if W.shape != ((d_in, d_out) if layout == 0 else (d_out, d_in)):
+        raise ValueError("W shape does not match the factors and layout")
+    out = np.zeros(W.shape, dtype=np.float64)
+    rc_ = lib.oracle_fold(d_in, d_out, rc, _ptr(At_c), _ptr(B_c), float(scale), _ptr(W), int(layout), _ptr(out))
+    if rc_ != 0:
+        raise ValueError(f"oracle_fold failed with {rc_}")
+    return out
 
 
 def adapter_bytes(d_in, d_out, rank: int) -> int:

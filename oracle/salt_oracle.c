@@ -29,11 +29,24 @@
  * -1 first, ties kept in token order; a domain segment is a maximal run of
  * equal domain and a user segment a maximal run of equal (domain, slot).
  *
+ * gamma (same section): the centroid of a request is scaled by a
+ * per-request coefficient taken from a few predefined bins, and requests are
+ * grouped by their (centroid, gamma) pair.  Here gamma is a per-token factor
+ * on the centroid term (1 when absent), and the grouping key is
+ * (domain, gamma bin, slot); a token without a centroid has no bin.
+ *
+ * Also here: the alignment regulariser of Phase 1 (Eq. 2), a matrix cosine
+ * between a task update Delta W and the centroid Wbar, evaluated from the
+ * dense matrices entry by entry; and the fold of a scaled centroid into a
+ * base weight (same section: high-frequency centroids are fused into the
+ * base weights at node startup), W + gamma * s_c * A_c B_c entry by entry.
+ *
  * All functions here are pinned by tests/test_oracle_pins.py against the
  * dense closed form, the concatenation identity, special cases, invariants,
- * a library sort, a hand-worked example and the paper's printed adapter
- * footprints.
+ * a library sort, a hand-worked example, the paper's printed adapter
+ * footprints, rank-one closed forms and dense brute force.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -53,6 +66,7 @@ static double oracle_bf16_value(uint16_t h)
  * x      [T][d_in]  bf16 bits, row-major
  * y_in   [T][d_out] bf16 bits (may be NULL: zeros)
  * dom    [T] centroid index or -1;  slot [T] residual slot or -1
+ * gamma  [T] per-token factor on the centroid term (NULL: 1 for every token)
  * For domain d: rc[d] ranks, s_c[d], At_c[d] -> [rc][d_in], B_c[d] -> [rc][d_out]
  * For slot u:   r_u[u] ranks, s_u[u], At_u[u] -> [r][d_in],  B_u[u] -> [r][d_out]
  * rows   [n_rows] token indices to evaluate (NULL: all T tokens in order)
@@ -61,7 +75,7 @@ static double oracle_bf16_value(uint16_t h)
  */
 int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
                  const uint16_t *x, const uint16_t *y_in,
-                 const int32_t *dom, const int32_t *slot,
+                 const int32_t *dom, const int32_t *slot, const double *gamma,
                  int32_t n_domains, const int32_t *rc, const double *s_c,
                  const uint16_t *const *At_c, const uint16_t *const *B_c,
                  int32_t n_slots, const int32_t *r_u, const double *s_u,
@@ -90,9 +104,10 @@ int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
         for (int64_t j = 0; j < d_out; ++j)
             out[j] = y_in ? oracle_bf16_value(y_in[t * d_out + j]) : 0.0;
 
-        /* centroid term: s_c * (x A_c) B_c */
+        /* centroid term: gamma * s_c * (x A_c) B_c */
         if (d >= 0) {
             int32_t R = rc[d];
+            double gt = gamma ? gamma[t] : 1.0;
             for (int32_t k = 0; k < R; ++k) {
                 double acc = 0.0;
                 for (int64_t i = 0; i < d_in; ++i)
@@ -103,7 +118,7 @@ int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
                 double acc = 0.0;
                 for (int32_t k = 0; k < R; ++k)
                     acc += v[k] * oracle_bf16_value(B_c[d][k * d_out + j]);
-                out[j] += s_c[d] * acc;
+                out[j] += gt * s_c[d] * acc;
             }
         }
         /* residual term: s_u * (x a_u) b_u */
@@ -131,29 +146,34 @@ int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
 /* Grouping of a heterogeneous batch into domain and user segments.        */
 
 typedef struct {
-    int32_t d, u, t;
+    int32_t d, g, u, t;
 } oracle_key;
 
 static int oracle_key_cmp(const void *pa, const void *pb)
 {
     const oracle_key *a = (const oracle_key *)pa, *b = (const oracle_key *)pb;
     if (a->d != b->d) return a->d < b->d ? -1 : 1;
+    if (a->g != b->g) return a->g < b->g ? -1 : 1;
     if (a->u != b->u) return a->u < b->u ? -1 : 1;
     if (a->t != b->t) return a->t < b->t ? -1 : 1;
     return 0;
 }
 
 /*
+ * gbin      [T]      gamma bin of each token, or NULL (no bins); the bin of
+ *                    a token without a centroid (dom = -1) is taken as -1
  * perm      [T]      token index of the i-th token in grouped order
- * dseg_ptr  [T + 1]  domain segment i spans [dseg_ptr[i], dseg_ptr[i+1])
- * dseg_dom  [T]      its domain
- * useg_ptr  [T + 1]  user segment i spans [useg_ptr[i], useg_ptr[i+1])
- * useg_dom, useg_slot [T]  its (domain, slot)
+ * dseg_ptr  [T + 1]  domain segment i spans [dseg_ptr[i], dseg_ptr[i+1]):
+ *                    a maximal run of equal (domain, bin)
+ * dseg_dom, dseg_gbin [T]  its (domain, bin)
+ * useg_ptr  [T + 1]  user segment i spans [useg_ptr[i], useg_ptr[i+1]):
+ *                    a maximal run of equal (domain, bin, slot)
+ * useg_dom, useg_gbin, useg_slot [T]  its (domain, bin, slot)
  * counts    [2]      number of domain segments, number of user segments
  */
-int oracle_segments(int32_t T, const int32_t *dom, const int32_t *slot,
-                    int32_t *perm, int32_t *dseg_ptr, int32_t *dseg_dom,
-                    int32_t *useg_ptr, int32_t *useg_dom, int32_t *useg_slot,
+int oracle_segments(int32_t T, const int32_t *dom, const int32_t *gbin, const int32_t *slot,
+                    int32_t *perm, int32_t *dseg_ptr, int32_t *dseg_dom, int32_t *dseg_gbin,
+                    int32_t *useg_ptr, int32_t *useg_dom, int32_t *useg_gbin, int32_t *useg_slot,
                     int32_t *counts)
 {
     oracle_key *keys;
@@ -169,20 +189,24 @@ int oracle_segments(int32_t T, const int32_t *dom, const int32_t *slot,
     if (!keys) return -2;
     for (int32_t t = 0; t < T; ++t) {
         keys[t].d = dom[t];
+        keys[t].g = (gbin && dom[t] >= 0) ? gbin[t] : -1;
         keys[t].u = slot[t];
         keys[t].t = t;
     }
     qsort(keys, (size_t)T, sizeof(oracle_key), oracle_key_cmp);
     for (int32_t i = 0; i < T; ++i) {
         perm[i] = keys[i].t;
-        if (i == 0 || keys[i].d != keys[i - 1].d) {
+        int new_dom = i == 0 || keys[i].d != keys[i - 1].d || keys[i].g != keys[i - 1].g;
+        if (new_dom) {
             dseg_ptr[nd] = i;
             dseg_dom[nd] = keys[i].d;
+            dseg_gbin[nd] = keys[i].g;
             ++nd;
         }
-        if (i == 0 || keys[i].d != keys[i - 1].d || keys[i].u != keys[i - 1].u) {
+        if (new_dom || keys[i].u != keys[i - 1].u) {
             useg_ptr[nu] = i;
             useg_dom[nu] = keys[i].d;
+            useg_gbin[nu] = keys[i].g;
             useg_slot[nu] = keys[i].u;
             ++nu;
         }
@@ -207,4 +231,84 @@ int64_t oracle_adapter_bytes(int32_t n_layers, const int32_t *d_in, const int32_
     for (int32_t l = 0; l < n_layers; ++l)
         params += (int64_t)rank * ((int64_t)d_in[l] + (int64_t)d_out[l]);
     return params * 2;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Phase 1 alignment regulariser (Eq. 2).                                  */
+
+/*
+ * L_align(Delta W, Wbar) = 1 - Tr(Delta W^T Wbar) / (||Delta W||_F ||Wbar||_F + eps)
+ * with Delta W = s * A B (rank r) and Wbar = s_c * A_c B_c (rank rc), both
+ * d_in x d_out, the A factors stored transposed (At[k][i]).  Evaluated from
+ * the dense matrices: each row i of both is formed in doubles and its
+ * entries enter the trace and the two squared norms.
+ *
+ * out[0] = L_align, out[1] = the cosine term Tr / (norms + eps),
+ * out[2] = Tr(Delta W^T Wbar), out[3] = ||Delta W||_F, out[4] = ||Wbar||_F.
+ */
+int oracle_align_loss(int64_t d_in, int64_t d_out,
+                      int32_t r, const uint16_t *At, const uint16_t *B, double s,
+                      int32_t rc, const uint16_t *At_c, const uint16_t *B_c, double s_c,
+                      double eps, double *out)
+{
+    double *dw = (double *)malloc(sizeof(double) * (size_t)(d_out > 0 ? d_out : 1));
+    double *wb = (double *)malloc(sizeof(double) * (size_t)(d_out > 0 ? d_out : 1));
+    double tr = 0.0, nn_dw = 0.0, nn_wb = 0.0;
+    if (!dw || !wb) {
+        free(dw);
+        free(wb);
+        return -2;
+    }
+    for (int64_t i = 0; i < d_in; ++i) {
+        for (int64_t j = 0; j < d_out; ++j) {
+            double a = 0.0, c = 0.0;
+            for (int32_t k = 0; k < r; ++k)
+                a += oracle_bf16_value(At[k * d_in + i]) * oracle_bf16_value(B[k * d_out + j]);
+            for (int32_t k = 0; k < rc; ++k)
+                c += oracle_bf16_value(At_c[k * d_in + i]) * oracle_bf16_value(B_c[k * d_out + j]);
+            dw[j] = s * a;
+            wb[j] = s_c * c;
+        }
+        for (int64_t j = 0; j < d_out; ++j) {
+            tr += dw[j] * wb[j];
+            nn_dw += dw[j] * dw[j];
+            nn_wb += wb[j] * wb[j];
+        }
+    }
+    free(dw);
+    free(wb);
+    {
+        double n_dw = sqrt(nn_dw), n_wb = sqrt(nn_wb);
+        double cosine = tr / (n_dw * n_wb + eps);
+        out[0] = 1.0 - cosine;
+        out[1] = cosine;
+        out[2] = tr;
+        out[3] = n_dw;
+        out[4] = n_wb;
+    }
+    return 0;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Fold of a scaled centroid into a base weight.                          */
+
+/*
+ * W_out = W + scale * A_c B_c entry by entry, in doubles (scale = gamma * s_c).
+ * layout 0: W is [d_in][d_out] (y = x W, the row-vector convention above);
+ * layout 1: W is [d_out][d_in] (y = x W^T, the weight of a linear layer).
+ * W holds bf16 bits; W_out gets the unrounded doubles in W's layout.
+ */
+int oracle_fold(int64_t d_in, int64_t d_out, int32_t rc, const uint16_t *At_c, const uint16_t *B_c,
+                double scale, const uint16_t *W, int32_t layout, double *W_out)
+{
+    if (layout != 0 && layout != 1) return -1;
+    for (int64_t i = 0; i < d_in; ++i)
+        for (int64_t j = 0; j < d_out; ++j) {
+            double acc = 0.0;
+            int64_t idx = layout ? j * d_in + i : i * d_out + j;
+            for (int32_t k = 0; k < rc; ++k)
+                acc += oracle_bf16_value(At_c[k * d_in + i]) * oracle_bf16_value(B_c[k * d_out + j]);
+            W_out[idx] = oracle_bf16_value(W[idx]) + scale * acc;
+        }
+    return 0;
 }

@@ -53,16 +53,17 @@ def _random_problem(wl, seed, T=16, d_in=48, d_out=40, n_dom=3, rcs=(8, 4, 0), n
     return x, y_in, dom, slot, cents, res
 
 
-def _dense_reference(x, y_in, dom, slot, cents, res):
-    """Closed form: materialise W_delta = s_c A_c B_c + s_u a_u b_u per token
-    as a d_in x d_out matrix of doubles and multiply."""
+def _dense_reference(x, y_in, dom, slot, cents, res, gamma=None):
+    """Closed form: materialise W_delta = gamma s_c A_c B_c + s_u a_u b_u per
+    token as a d_in x d_out matrix of doubles and multiply."""
     xv, yv = _val(x), _val(y_in)
     out = yv.copy()
     for t in range(x.shape[0]):
         W = np.zeros((x.shape[1], y_in.shape[1]))
         if dom[t] >= 0:
             A, B, s = cents[dom[t]]
-            W += s * (_val(A).T @ _val(B))
+            g = 1.0 if gamma is None else gamma[t]
+            W += (g * s) * (_val(A).T @ _val(B))
         if slot[t] >= 0:
             A, B, s = res[slot[t]]
             W += s * (_val(A).T @ _val(B))
@@ -85,6 +86,21 @@ def test_dense_closed_form(oracle_mod, wl, seed):
     got = oracle_mod.apply(x, y_in, dom, slot, cents, res)
     scale = np.abs(ref).max()
     assert np.abs(got - ref).max() <= 1e-12 * scale
+
+
+@pytest.mark.parametrize("seed", [20, 21])
+def test_dense_closed_form_with_gamma(oracle_mod, wl, seed):
+    """W_final = W_base + gamma Wbar + delta_i with a per-request gamma from
+    the bins {0.6, 0.8, 1.0} (Section "Multi-Tenant Serving")."""
+    x, y_in, dom, slot, cents, res = _random_problem(wl, seed)
+    bins = np.array([0.6, 0.8, 1.0])
+    gamma = bins[(wl.uniform(seed, wl.stream_id(99, 40), x.shape[0]) * 3).astype(int) % 3]
+    ref = _dense_reference(x, y_in, dom, slot, cents, res, gamma)
+    got = oracle_mod.apply(x, y_in, dom, slot, cents, res, gamma=gamma)
+    assert np.abs(got - ref).max() <= 1e-12 * np.abs(ref).max()
+    # gamma = 1 everywhere is the plain result, bit for bit
+    np.testing.assert_array_equal(oracle_mod.apply(x, y_in, dom, slot, cents, res, gamma=np.ones(x.shape[0])),
+                                  oracle_mod.apply(x, y_in, dom, slot, cents, res))
 
 
 def test_dense_closed_form_config0_shape(oracle_mod, wl):
@@ -282,3 +298,140 @@ def test_sixteen_fold_swap_reduction(oracle_mod):
     """Abstract / introduction: a rank-16 adapter swaps 16x the bytes of rank 1."""
     din, dout = [4096, 4096] * 32, [4096, 1024] * 32
     assert oracle_mod.adapter_bytes(din, dout, 16) == 16 * oracle_mod.adapter_bytes(din, dout, 1)
+
+
+# ---------------------------------------------------------------- grouping by (centroid, gamma)
+def _check_gamma_segments_against_lexsort(s, dom, gbin, slot):
+    """Stable order of (domain, bin, slot) with the bin of a centroid-less
+    token taken as -1; runs of equal (domain, bin) and (domain, bin, slot)."""
+    T = len(dom)
+    g = np.where(dom >= 0, gbin, -1)
+    order = np.lexsort((np.arange(T), slot, g, dom))
+    np.testing.assert_array_equal(s["perm"], order)
+    sd, sg, su = dom[order], g[order], slot[order]
+    if T:
+        dchg = (sd[1:] != sd[:-1]) | (sg[1:] != sg[:-1])
+        dh = np.flatnonzero(np.r_[True, dchg])
+        uh = np.flatnonzero(np.r_[True, dchg | (su[1:] != su[:-1])])
+    else:
+        dh = uh = np.array([], dtype=int)
+    np.testing.assert_array_equal(s["dseg_ptr"], np.r_[dh, T])
+    np.testing.assert_array_equal(s["dseg_dom"], sd[dh])
+    np.testing.assert_array_equal(s["dseg_gbin"], sg[dh])
+    np.testing.assert_array_equal(s["useg_ptr"], np.r_[uh, T])
+    np.testing.assert_array_equal(s["useg_dom"], sd[uh])
+    np.testing.assert_array_equal(s["useg_gbin"], sg[uh])
+    np.testing.assert_array_equal(s["useg_slot"], su[uh])
+
+
+@pytest.mark.parametrize("T,nd,ng,ns", [(1, 1, 1, 1), (50, 3, 3, 7), (2000, 8, 4, 300)])
+def test_gamma_segments_match_library_sort(oracle_mod, wl, T, nd, ng, ns):
+    dom = (wl.uniform(T, wl.stream_id(98, 11), T) * (nd + 1)).astype(np.int32) - 1
+    gbin = (wl.uniform(T, wl.stream_id(98, 12), T) * (ng + 1)).astype(np.int32) - 1
+    slot = (wl.uniform(T, wl.stream_id(98, 13), T) * (ns + 1)).astype(np.int32) - 1
+    _check_gamma_segments_against_lexsort(oracle_mod.segments(dom, slot, gbin), dom, gbin, slot)
+
+
+def test_gamma_segments_exhaustive_tiny(oracle_mod):
+    """Brute force: every 3-token batch with domain, bin in {-1, 0, 1} and slot in {-1, 0}."""
+    import itertools
+    for d in itertools.product((-1, 0, 1), repeat=3):
+        for g in itertools.product((-1, 0, 1), repeat=3):
+            for u in itertools.product((-1, 0), repeat=3):
+                dom, gbin, slot = (np.array(v, dtype=np.int32) for v in (d, g, u))
+                _check_gamma_segments_against_lexsort(oracle_mod.segments(dom, slot, gbin), dom, gbin, slot)
+
+
+def test_gamma_segments_without_bins_are_plain(oracle_mod, wl):
+    T = 300
+    dom = (wl.uniform(3, wl.stream_id(98, 21), T) * 5).astype(np.int32) - 1
+    slot = (wl.uniform(3, wl.stream_id(98, 22), T) * 9).astype(np.int32) - 1
+    a = oracle_mod.segments(dom, slot)
+    b = oracle_mod.segments(dom, slot, np.zeros(T, np.int32))
+    for k in ("perm", "dseg_ptr", "dseg_dom", "useg_ptr", "useg_dom", "useg_slot"):
+        np.testing.assert_array_equal(a[k], b[k], err_msg=k)
+    assert set(a["dseg_gbin"].tolist()) == {-1}
+
+
+# ---------------------------------------------------------------- alignment regulariser (Eq. 2)
+def _factors(wl, seed, r, rc, d_in, d_out):
+    sid = wl.stream_id
+    At = wl.normal_bf16(seed, sid(97, 1), r * d_in, 1 / np.sqrt(d_in)).reshape(r, d_in)
+    B = wl.normal_bf16(seed, sid(97, 2), r * d_out, 1 / np.sqrt(max(r, 1))).reshape(r, d_out)
+    Atc = wl.normal_bf16(seed, sid(97, 3), rc * d_in, 1 / np.sqrt(d_in)).reshape(rc, d_in)
+    Bc = wl.normal_bf16(seed, sid(97, 4), rc * d_out, 1 / np.sqrt(max(rc, 1))).reshape(rc, d_out)
+    return At, B, Atc, Bc
+
+
+@pytest.mark.parametrize("seed,r,rc,d_in,d_out,s,s_c", [(0, 2, 8, 24, 40, 1.0, 1.0), (1, 1, 16, 64, 16, 2.0, -0.5),
+                                                        (2, 4, 3, 8, 8, 0.25, 3.0)])
+def test_align_dense_brute_force(oracle_mod, wl, seed, r, rc, d_in, d_out, s, s_c):
+    At, B, Atc, Bc = _factors(wl, seed, r, rc, d_in, d_out)
+    got = oracle_mod.align_loss(At, B, s, Atc, Bc, s_c, eps=1e-8)
+    dW = s * (_val(At).T @ _val(B))
+    Wb = s_c * (_val(Atc).T @ _val(Bc))
+    tr = float(np.sum(dW * Wb))
+    n1, n2 = float(np.linalg.norm(dW)), float(np.linalg.norm(Wb))
+    assert abs(got["trace"] - tr) <= 1e-12 * n1 * n2
+    assert abs(got["norm_dw"] - n1) <= 1e-12 * n1 and abs(got["norm_wbar"] - n2) <= 1e-12 * n2
+    assert abs(got["loss"] - (1 - tr / (n1 * n2 + 1e-8))) <= 1e-12
+
+
+def test_align_rank_one_closed_form(oracle_mod, wl):
+    """Delta W = a b^T, Wbar = a' b'^T: the matrix cosine is the product of the
+    two vector cosines, cos(a, a') cos(b, b')."""
+    At, B, Atc, Bc = _factors(wl, 5, 1, 1, 96, 40)
+    got = oracle_mod.align_loss(At, B, 1.0, Atc, Bc, 1.0, eps=0.0)
+    a, b, a2, b2 = (_val(v)[0] for v in (At, B, Atc, Bc))
+    cos = (a @ a2) / np.linalg.norm(a) / np.linalg.norm(a2) * (b @ b2) / np.linalg.norm(b) / np.linalg.norm(b2)
+    assert abs(got["cosine"] - cos) <= 1e-13
+    assert abs(got["loss"] - (1 - cos)) <= 1e-13
+
+
+def test_align_special_cases(oracle_mod, wl):
+    At, B, Atc, Bc = _factors(wl, 6, 2, 5, 32, 24)
+    # the centroid itself: cosine 1 up to eps
+    same = oracle_mod.align_loss(Atc, Bc, 1.0, Atc, Bc, 1.0)
+    assert abs(same["loss"]) <= 1e-7
+    # its negation: loss 2
+    neg = oracle_mod.align_loss(Atc, Bc, -1.0, Atc, Bc, 1.0)
+    assert abs(neg["loss"] - 2.0) <= 1e-7
+    # a zero centroid: the trace is 0 and eps keeps the quotient finite: loss exactly 1
+    zero = oracle_mod.align_loss(At, B, 1.0, np.zeros_like(Atc), Bc, 1.0)
+    assert zero["loss"] == 1.0 and zero["trace"] == 0.0
+    # disjoint input supports: Delta W and Wbar have no common nonzero entry: loss exactly 1
+    A1, A2 = At.copy(), Atc.copy()
+    A1[:, 16:] = 0
+    A2[:, :16] = 0
+    dis = oracle_mod.align_loss(A1, B, 1.0, A2, Bc, 1.0)
+    assert dis["trace"] == 0.0 and dis["loss"] == 1.0
+    # positive scales leave the cosine unchanged (up to eps)
+    a = oracle_mod.align_loss(At, B, 1.0, Atc, Bc, 1.0, eps=0.0)
+    b = oracle_mod.align_loss(At, B, 4.0, Atc, Bc, 0.5, eps=0.0)
+    assert abs(a["cosine"] - b["cosine"]) <= 1e-14
+
+
+# ---------------------------------------------------------------- centroid fold
+@pytest.mark.parametrize("layout", [0, 1])
+def test_fold_dense_brute_force(oracle_mod, wl, layout):
+    At, B, Atc, Bc = _factors(wl, 7, 1, 6, 40, 24)
+    W = wl.normal_bf16(7, wl.stream_id(97, 9), 40 * 24).reshape(40, 24)
+    Wl = W if layout == 0 else np.ascontiguousarray(W.T)
+    got = oracle_mod.fold(Atc, Bc, 0.7, Wl, layout)
+    ref = _val(W) + 0.7 * (_val(Atc).T @ _val(Bc))
+    if layout:
+        ref = ref.T
+    assert np.abs(got - ref).max() <= 1e-13 * np.abs(ref).max()
+
+
+def test_fold_special_cases(oracle_mod, wl):
+    At, B, Atc, Bc = _factors(wl, 8, 1, 4, 16, 32)
+    W = wl.normal_bf16(8, wl.stream_id(97, 10), 16 * 32).reshape(16, 32)
+    np.testing.assert_array_equal(oracle_mod.fold(Atc, Bc, 0.0, W, 0), _val(W))
+    # the two layouts hold the same matrix, transposed
+    a = oracle_mod.fold(Atc, Bc, -1.25, W, 0)
+    b = oracle_mod.fold(Atc, Bc, -1.25, np.ascontiguousarray(W.T), 1)
+    np.testing.assert_array_equal(a, b.T)
+    # fold then unfold returns W (in doubles, before any rounding)
+    delta = oracle_mod.fold(Atc, Bc, 0.8, np.zeros_like(W), 0)
+    assert np.abs((a - _val(W)) + 1.25 / 0.8 * delta).max() <= 1e-13 * np.abs(delta).max()
