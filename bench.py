@@ -17,6 +17,15 @@ trained checkpoint.  `value` is tokens/s with x / y resident in HBM; `e2e`
 adds the host <-> device copies of x, y_in and y to every step.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--mode salt|rank16]
+                  [--gamma-bins] [--row fold|align]
+
+--gamma-bins groups the same step by (centroid, gamma bin), each token in
+one of the bins 0.6 / 0.8 / 1.0 (salt_build_segments_gamma).  --row prints
+the line of another part of the path instead of the step: `fold` fuses one
+domain's rank-64 centroid into all 224 adapted weights of the 32 layers
+(salt_centroid_fold, alternating +gamma and -gamma), `align` evaluates the
+alignment regulariser over the same 224 matrices for a rank-16 task update
+against the rank-64 centroid (salt_align_loss).
 
 Under torchrun (N > 1) every rank runs an independent replica on its own
 GPU (the path has no exchange step); rank 0 prints one JSON line.
@@ -55,6 +64,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--gamma-bins", action="store_true")
+    ap.add_argument("--row", default="step", choices=["step", "fold", "align"])
     return ap.parse_args()
 
 
@@ -193,6 +204,8 @@ class Step:
         self.L = len(self.w.layers)
         self.groups = groups_of(args.layers)
         self.ids = [wl.config4_ids(4, s, self.T) for s in range(self.N_ID_SETS)]
+        self.gbins = ([wl.gamma_bin_ids(4 + s, self.T) for s in range(self.N_ID_SETS)]
+                      if getattr(args, "gamma_bins", False) else None)
         if rank16:
             self.ids = [(np.full(self.T, -1, np.int32), sl) for (_, sl) in self.ids]
         self.runner = SaltRunner(self.w, device=device, max_tokens=self.T)
@@ -252,7 +265,11 @@ class Step:
 
     def build(self, s):
         dom, slot = self.ids[s % self.N_ID_SETS]
-        self.salt.salt_build_segments(self.runner.ctx, self.runner.seg, dom, slot, stream=self.comp)
+        if self.gbins is not None:
+            self.salt.salt_build_segments_gamma(self.runner.ctx, self.runner.seg, dom, self.gbins[s % self.N_ID_SETS],
+                                                slot, self.wl_mod.GAMMA_BINS, stream=self.comp)
+        else:
+            self.salt.salt_build_segments(self.runner.ctx, self.runner.seg, dom, slot, stream=self.comp)
 
     def applies_eager(self, timing=False):
         torch = self.torch
@@ -558,7 +575,8 @@ def run_salt(args, rank, world, local, pg):
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": WORKLOAD if args.mode == "salt" else WORKLOAD + "_rank16_lora",
+                "config": {"workload": (WORKLOAD if args.mode == "salt" else WORKLOAD + "_rank16_lora")
+                           + ("_gamma_bins" if args.gamma_bins else ""),
                            "tokens_per_step": st.T, "layers": args.layers, "projections": st.L,
                            "domains": 8, "centroid_rank": 0 if args.mode == "rank16" else 64,
                            "residual_rank": 16 if args.mode == "rank16" else 2, "slots": 512,
@@ -576,6 +594,102 @@ def run_salt(args, rank, world, local, pg):
         print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------------------------- other rows of the path
+def run_row(args, rank, world, local, pg):
+    """One JSON line for the centroid fold or the alignment regulariser over
+    the 224 adapted matrices of Llama-3.1-8B (32 layers x q, k, v, o, gate,
+    up, down), timed with CUDA events on the launching stream."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_03579_gb300 import salt
+    from paper_2608_03579_gb300 import workloads as wl
+    torch.cuda.set_device(local)
+    peaks, peak_kind = load_peaks()
+    shapes = [(din, dout) for _ in range(args.layers) for (_, din, dout) in wl.LLAMA8B_LAYER]
+    n = len(shapes)
+    stream = torch.cuda.Stream(device=local)
+    gen = torch.Generator(device=f"cuda:{local}")
+    gen.manual_seed(4)
+
+    def randn(*shape, std=1.0):
+        return (torch.randn(*shape, generator=gen, device=f"cuda:{local}") * std).to(torch.bfloat16)
+
+    rc = 64
+    if args.row == "fold":
+        d_in = [a for a, _ in shapes]
+        d_out = [b for _, b in shapes]
+        ctx = salt.salt_ctx_create(d_in, d_out, 1, rc, 1, 1, 16, local)
+        A = np.concatenate([wl.normal_bf16(4, wl.stream_id(wl.K_CENT_A, 0, l), rc * a, 1 / np.sqrt(a))
+                            for l, (a, _) in enumerate(shapes)])
+        B = np.concatenate([wl.normal_bf16(4, wl.stream_id(wl.K_CENT_B, 0, l), rc * b, 1 / np.sqrt(rc))
+                            for l, (_, b) in enumerate(shapes)])
+        salt.salt_centroid_pin(ctx, 0, rc, A, B, 1.0)
+        # base weights as a linear layer stores them, [d_out][d_in]
+        W = [randn(b, a, std=0.02) for (a, b) in shapes]
+        w_bytes = sum(a * b * 2 for a, b in shapes)
+        alg = 2 * w_bytes + sum(rc * (a + b) * 2 for a, b in shapes)
+
+        def one(k):
+            g = 0.8 if k % 2 == 0 else -0.8
+            for l in range(n):
+                salt.salt_centroid_fold(ctx, 0, l, g, W[l], salt.SALT_W_OUT_IN, stream)
+        metric, unit, what = "centroid fold GB/s (W += gamma s_c A_c B_c over every adapted weight)", "GB/s", \
+            "llama8b_32layer_centroid_fold_rank64"
+    else:
+        r = 16
+        keep, pairs = [], []
+        for (a, b) in shapes:
+            t = (randn(r, a, std=a ** -0.5), randn(r, b, std=r ** -0.5), randn(rc, a, std=a ** -0.5),
+                 randn(rc, b, std=rc ** -0.5))
+            keep.append(t)
+            pairs.append(dict(At=t[0], B=t[1], At_c=t[2], B_c=t[3], r=r, rc=rc, d_in=a, d_out=b, s=1.0, s_c=1.0))
+        loss = torch.empty(n, device=f"cuda:{local}")
+        alg = sum((r + rc) * (a + b) * 2 for a, b in shapes)
+        ctx = None
+
+        def one(k):
+            salt.salt_align_loss(pairs, 1e-8, loss, None, stream)
+        metric, unit, what = "alignment regulariser GB/s (Eq. 2, factored, every adapted weight)", "GB/s", \
+            "llama8b_32layer_align_rank16_vs_rank64"
+    for k in range(args.warmup):
+        one(k)
+    torch.cuda.synchronize(local)
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid, os.path.join(ROOT, "gpurun_out", f"clocks_{args.row}_rank{rank}.csv"))
+    barrier(pg, local)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with sampler:
+        time.sleep(0.2)
+        e0.record(stream)
+        for k in range(args.steps):
+            one(args.warmup + k)
+        e1.record(stream)
+        torch.cuda.synchronize(local)
+    ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / args.steps
+    achieved = alg / (ms / 1000.0) / 1e9
+    clocks = sampler.summary()
+    if ctx is not None:
+        salt.salt_ctx_destroy(ctx)
+    if rank == 0:
+        launches = n if args.row == "fold" else 2 * ((n + 31) // 32)
+        print(json.dumps({
+            "metric": metric, "value": world * achieved, "unit": unit, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": what, "matrices": n, "algorithmic_bytes_per_step": alg,
+                       "l2": "inputs larger than L2"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": achieved / peaks["hbm_gbs"], "traffic": None},
+            "gpu_launches": args.steps * launches,
+            "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")}}), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -584,7 +698,10 @@ def main():
         return
     rank, world, local, pg = dist_setup(args)
     try:
-        run_salt(args, rank, world, local, pg)
+        if args.row != "step":
+            run_row(args, rank, world, local, pg)
+        else:
+            run_salt(args, rank, world, local, pg)
     finally:
         if pg is not None:
             pg.destroy_process_group()

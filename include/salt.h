@@ -47,8 +47,11 @@ extern "C" {
 /* Library limits. */
 #define SALT_MAX_TOKENS 16384        /* tokens per segments build */
 #define SALT_MAX_CENTROID_RANK 64    /* rc_max */
-#define SALT_MAX_RESIDUAL_RANK 16    /* r_max (16 covers the rank-16 LoRA comparison) */
+#define SALT_MAX_RESIDUAL_RANK 80    /* r_max: up to a rank-64 centroid concatenated with a rank-16 residual */
+#define SALT_MAX_TOKEN_RANK 80       /* rc_max + r_max (a token's centroid plus residual rank) */
 #define SALT_MAX_GROUP 8             /* projections per grouped apply */
+#define SALT_MAX_GAMMA_BINS 16       /* gamma bins of one segments build */
+#define SALT_MAX_ALIGN_RANK 128      /* r + rc of one alignment pair */
 #define SALT_BLOB_HEADER_BYTES 256
 #define SALT_BLOB_MAGIC 0x3153455254414C53ULL /* "SALTRES1" little-endian */
 
@@ -74,7 +77,8 @@ typedef enum salt_status {
     SALT_ERR_TOO_MANY_TOKENS = 14,   /* n_tokens above the context's max_tokens */
     SALT_ERR_DOMAIN_RANGE = 15,      /* domain id outside [-1, n_domains) */
     SALT_ERR_STALE_SEGMENTS = 16,    /* a slot the segments read was reloaded after the build */
-    SALT_ERR_NOT_BUILT = 17          /* segments object was never built */
+    SALT_ERR_NOT_BUILT = 17,         /* segments object was never built */
+    SALT_ERR_GAMMA_RANGE = 18        /* gamma bin outside [-1, n_gamma) */
 } salt_status;
 
 /* Bits of the device error word (salt_get_device_error). */
@@ -84,12 +88,14 @@ typedef enum salt_status {
 #define SALT_DEVERR_SLOT_EMPTY 0x8u
 #define SALT_DEVERR_RANK 0x10u
 #define SALT_DEVERR_TIMEOUT 0x20u        /* a bounded in-kernel wait gave up (results of that call invalid) */
+#define SALT_DEVERR_GAMMA_RANGE 0x40u
 
 /*
  * Context configuration.  d_in / d_out are host arrays of n_layers entries,
  * each a positive multiple of 8 (16-byte rows).  rc_max <=
  * SALT_MAX_CENTROID_RANK, 1 <= r_max <= SALT_MAX_RESIDUAL_RANK,
- * rc_max + r_max <= 128, 1 <= max_tokens <= SALT_MAX_TOKENS.
+ * rc_max + r_max <= SALT_MAX_TOKEN_RANK, 1 <= max_tokens <= SALT_MAX_TOKENS,
+ * n_domains < 2^17 - 1, n_slots < 2^17.
  */
 typedef struct salt_config {
     int32_t n_layers;
@@ -115,7 +121,7 @@ typedef struct salt_config {
 typedef struct salt_blob_header {
     uint64_t magic;          /* SALT_BLOB_MAGIC */
     uint32_t version;        /* 1 */
-    int32_t rank;            /* 1 .. r_max */
+    int32_t rank;            /* 1 .. SALT_MAX_RESIDUAL_RANK (and <= r_max of the loading context) */
     int32_t n_layers;
     float s_u;               /* residual scale */
     uint64_t payload_bytes;
@@ -184,6 +190,47 @@ salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, flo
                                     void *blob, int64_t blob_bytes);
 
 /*
+ * The long-tail form of a request (Section "Multi-Tenant Serving": for rare
+ * tasks the scaled centroid and the residual are concatenated offline into
+ * one standard adapter, e.g. rank 17, served by plain heterogeneous
+ * batching): write a blob of rank rc + rank whose factors are, per layer,
+ *     At = [At_c ; At_u]           ([rc + rank][d_in_l])
+ *     B  = [(s_c / s) B_c ; B_u]   ([rc + rank][d_out_l])
+ * with blob scale s = s_u (s = 1 and B_u scaled by 0 when s_u == 0), so
+ * that s (x At^T) B = s_c (x A_c) B_c + s_u (x a_u) b_u.  At_c / B_c are
+ * host arrays in salt_centroid_pin's layout (rank rc), At_u / B_u in
+ * salt_residual_blob_pack's (rank `rank`); s_c is the centroid's scale
+ * with gamma applied.  The A rows are copied bit for bit; a scaled B row is
+ * rounded once to bf16 (round to nearest even) and copied bit for bit when
+ * s_c == s.  rc + rank <= SALT_MAX_RESIDUAL_RANK; the blob loads into a
+ * context whose r_max is at least that and is applied with domain id -1.
+ * Host only, synchronous.
+ */
+salt_status salt_residual_blob_concat(const salt_config *config, int32_t rc, const void *At_c,
+                                      const void *B_c, float s_c, int32_t rank, const void *At_u,
+                                      const void *B_u, float s_u, void *blob, int64_t blob_bytes);
+
+/*
+ * Fuse a scaled centroid into a base weight (Section "Multi-Tenant
+ * Serving": high-frequency centroids are fused into the base weights at
+ * node startup, after which their requests swap and apply only residuals:
+ * build their segments with domain id -1).  For layer `layer` and pinned
+ * domain `domain`:
+ *     W += gamma * s_c(domain) * A_c B_c
+ * in place, each element accumulated in fp32 and rounded once to bf16
+ * (round to nearest even).  W is device bf16, 16-byte aligned, in one of
+ *     SALT_W_IN_OUT: W[d_in][d_out]  (y = x W, this library's convention)
+ *     SALT_W_OUT_IN: W[d_out][d_in]  (y = x W^T, a linear layer's weight)
+ * gamma = -g undoes a fold by g up to the two roundings.  One tcgen05
+ * kernel; asynchronous on `stream`, after earlier work on it.  The
+ * centroid must not be re-pinned while the fold runs.
+ */
+#define SALT_W_IN_OUT 0
+#define SALT_W_OUT_IN 1
+salt_status salt_centroid_fold(salt_ctx *ctx, int32_t domain, int32_t layer, float gamma, void *W,
+                               int32_t layout, salt_stream_t stream);
+
+/*
  * Page-locked host memory for residual blobs, backed by transparent huge
  * pages where the kernel offers them (anonymous mapping rounded up to the
  * huge-page size, madvise(MADV_HUGEPAGE), every page touched, then
@@ -242,6 +289,33 @@ void salt_segments_destroy(salt_segments *seg);
 salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg,
                                  const int32_t *domain_ids, const int32_t *slot_ids,
                                  int32_t n_tokens, salt_stream_t stream);
+
+/*
+ * salt_build_segments with gamma bins (Section "Multi-Tenant Serving":
+ * gamma is discretised into a few predefined bins and the frontend groups
+ * requests by their (centroid, gamma) pair).  gamma_bins is int32[n_tokens]
+ * in the same kind of memory as the other ids; each entry is -1 (no gamma:
+ * the pinned s_c as is) or a bin in [0, n_gamma), and gamma[0..n_gamma)
+ * (host floats, 0 <= n_gamma <= SALT_MAX_GAMMA_BINS, read during the call)
+ * are the bins' values.  A token with domain d and bin g has the centroid
+ * scale s_c(d) * gamma[g]; a token without a centroid ignores its bin.
+ * Tokens are sorted stably by (domain, bin, slot), -1 first; domain runs
+ * become runs of equal (domain, bin) and user runs runs of equal (domain,
+ * bin, slot) (their bins: salt_segments_export_gamma).  A bin outside the
+ * range is SALT_ERR_GAMMA_RANGE for host ids, SALT_DEVERR_GAMMA_RANGE (and
+ * bin -1) for device ids.  Otherwise as salt_build_segments, which is this
+ * call with every bin -1.
+ */
+salt_status salt_build_segments_gamma(salt_ctx *ctx, salt_segments *seg, const int32_t *domain_ids,
+                                      const int32_t *gamma_bins, const int32_t *slot_ids,
+                                      int32_t n_tokens, int32_t n_gamma, const float *gamma,
+                                      salt_stream_t stream);
+
+/* The gamma bins of the last build's domain runs and user runs (-1: none),
+ * in the order of salt_segments_export's dseg_* and useg_* arrays.  Either
+ * pointer may be NULL.  Synchronous. */
+salt_status salt_segments_export_gamma(salt_ctx *ctx, const salt_segments *seg, int32_t *dseg_gbin,
+                                       int32_t *useg_gbin);
 
 /*
  * Copy the segment metadata to host buffers (synchronous; for tests and
@@ -304,6 +378,35 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
  */
 salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
                                    const void *x, void *y, salt_stream_t stream);
+
+/*
+ * The alignment regulariser of Phase 1 (Eq. 2), for n pairs of a task
+ * update and a centroid:
+ *     L_align = 1 - Tr(dW^T Wbar) / (||dW||_F ||Wbar||_F + eps),
+ *     dW = s A B (rank r),  Wbar = s_c A_c B_c (rank rc),
+ * evaluated without forming either d_in x d_out matrix: with the stacked
+ * factors F_in = [At ; At_c] ([r + rc][d_in]) and F_out = [B ; B_c], the
+ * trace and both squared norms are sums over blocks of G_in o G_out, where
+ * G = F F^T are (r + rc)^2 Gram matrices contracted on the tensor cores
+ * (bf16 operands, fp32 accumulation) and combined in fp64.  The paper's
+ * eps is 1e-8.  pairs is a host array; its factor pointers are device bf16
+ * arrays, rows contiguous, 16-byte aligned; 1 <= r, 1 <= rc,
+ * r + rc <= SALT_MAX_ALIGN_RANK, d_in and d_out positive multiples of 8.
+ * loss and cosine (the quotient; may be NULL) are device float[n].
+ * Scratch comes from the stream-ordered allocator of the current device.
+ * Asynchronous on `stream`.  Not on the serving path: the regulariser of
+ * centroid training, offered for checking or monitoring alignment.
+ */
+typedef struct salt_align_pair {
+    const void *At;     /* [r][d_in]   task update's A, transposed */
+    const void *B;      /* [r][d_out]  task update's B */
+    const void *At_c;   /* [rc][d_in]  centroid's A, transposed */
+    const void *B_c;    /* [rc][d_out] centroid's B */
+    int32_t r, rc, d_in, d_out;
+    float s, s_c;       /* scales of dW and Wbar */
+} salt_align_pair;
+salt_status salt_align_loss(int32_t n, const salt_align_pair *pairs, float eps, float *loss,
+                            float *cosine, salt_stream_t stream);
 
 /*
  * Self-test of the failure path.  Enqueues on `stream` one thread that

@@ -260,14 +260,19 @@ int oracle_align_loss(int64_t d_in, int64_t d_out,
         return -2;
     }
     for (int64_t i = 0; i < d_in; ++i) {
+        /* row i of A B and of A_c B_c, summed over k in ascending order */
+        for (int64_t j = 0; j < d_out; ++j) dw[j] = wb[j] = 0.0;
+        for (int32_t k = 0; k < r; ++k) {
+            double a = oracle_bf16_value(At[k * d_in + i]);
+            for (int64_t j = 0; j < d_out; ++j) dw[j] += a * oracle_bf16_value(B[k * d_out + j]);
+        }
+        for (int32_t k = 0; k < rc; ++k) {
+            double c = oracle_bf16_value(At_c[k * d_in + i]);
+            for (int64_t j = 0; j < d_out; ++j) wb[j] += c * oracle_bf16_value(B_c[k * d_out + j]);
+        }
         for (int64_t j = 0; j < d_out; ++j) {
-            double a = 0.0, c = 0.0;
-            for (int32_t k = 0; k < r; ++k)
-                a += oracle_bf16_value(At[k * d_in + i]) * oracle_bf16_value(B[k * d_out + j]);
-            for (int32_t k = 0; k < rc; ++k)
-                c += oracle_bf16_value(At_c[k * d_in + i]) * oracle_bf16_value(B_c[k * d_out + j]);
-            dw[j] = s * a;
-            wb[j] = s_c * c;
+            dw[j] *= s;
+            wb[j] *= s_c;
         }
         for (int64_t j = 0; j < d_out; ++j) {
             tr += dw[j] * wb[j];
@@ -301,14 +306,24 @@ int oracle_align_loss(int64_t d_in, int64_t d_out,
 int oracle_fold(int64_t d_in, int64_t d_out, int32_t rc, const uint16_t *At_c, const uint16_t *B_c,
                 double scale, const uint16_t *W, int32_t layout, double *W_out)
 {
-    if (layout != 0 && layout != 1) return -1;
-    for (int64_t i = 0; i < d_in; ++i)
-        for (int64_t j = 0; j < d_out; ++j) {
-            double acc = 0.0;
-            int64_t idx = layout ? j * d_in + i : i * d_out + j;
-            for (int32_t k = 0; k < rc; ++k)
-                acc += oracle_bf16_value(At_c[k * d_in + i]) * oracle_bf16_value(B_c[k * d_out + j]);
-            W_out[idx] = oracle_bf16_value(W[idx]) + scale * acc;
+    double *row = (double *)malloc(sizeof(double) * (size_t)(d_out > 0 ? d_out : 1));
+    if (layout != 0 && layout != 1) {
+        free(row);
+        return -1;
+    }
+    if (!row) return -2;
+    for (int64_t i = 0; i < d_in; ++i) {
+        /* row i of A_c B_c, summed over k in ascending order */
+        for (int64_t j = 0; j < d_out; ++j) row[j] = 0.0;
+        for (int32_t k = 0; k < rc; ++k) {
+            double a = oracle_bf16_value(At_c[k * d_in + i]);
+            for (int64_t j = 0; j < d_out; ++j) row[j] += a * oracle_bf16_value(B_c[k * d_out + j]);
         }
+        for (int64_t j = 0; j < d_out; ++j) {
+            int64_t idx = layout ? j * d_in + i : i * d_out + j;
+            W_out[idx] = oracle_bf16_value(W[idx]) + scale * row[j];
+        }
+    }
+    free(row);
     return 0;
 }

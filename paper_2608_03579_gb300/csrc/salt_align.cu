@@ -1,0 +1,325 @@
+// The alignment regulariser of Phase 1 (Eq. 2) in factored form.
+//
+//     L_align = 1 - Tr(dW^T Wbar) / (||dW||_F ||Wbar||_F + eps),
+//     dW = s A B (rank r),   Wbar = s_c A_c B_c (rank rc)
+//
+// Neither d_in x d_out matrix is formed.  With the stacked factors
+// F_in = [At ; At_c] ([r + rc][d_in]) and F_out = [B ; B_c] ([r + rc][d_out])
+// and their Gram matrices G = F F^T,
+//     Tr(dW^T Wbar) = s s_c sum_{k < r, l >= r} G_in[k][l] G_out[k][l]
+//     ||dW||_F^2    = s^2   sum_{k, l < r}      G_in[k][l] G_out[k][l]
+//     ||Wbar||_F^2  = s_c^2 sum_{k, l >= r}     G_in[k][l] G_out[k][l]
+// so the work is two Gram contractions per pair, each a pass over its
+// factors: HBM-bound, (r + rc)(d_in + d_out) bf16 read once.
+//
+// align_gram_kernel: one CTA per unit (pair, side, K-split); the unit's
+// 64-column chunks of F stream through a cp.async ring into a 128-byte-
+// swizzled K-major tile that is both operands of tcgen05.mma
+// (D[128 x S] += F_chunk F_chunk^T, fp32 in tensor memory); the unit writes
+// its S x S partial.  align_combine_kernel: one CTA per pair sums the
+// partials of each side over the splits in split order (fp32), forms the
+// three block sums of G_in o G_out in fp64 and writes the loss.
+#include "salt_async.cuh"
+#include "salt_internal.cuh"
+#include "salt_tcgen05.cuh"
+
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+namespace salt {
+namespace {
+
+constexpr int ALIGN_THREADS = 128;
+constexpr int ALIGN_STAGES = 4;
+constexpr int ALIGN_STAGE_BYTES = 128 * 128;     // <= 128 stacked rows x 64 columns
+constexpr int ALIGN_SMEM = 1024 + ALIGN_STAGES * ALIGN_STAGE_BYTES;
+constexpr int ALIGN_MAX_PAIRS = 32;              // pairs per launch
+constexpr int ALIGN_PART = 128 * 128;            // floats per unit partial (row pitch S)
+constexpr int COMBINE_THREADS = 256;
+static_assert(SALT_MAX_ALIGN_RANK <= 128, "a stack is the 128-row UMMA operand");
+
+struct AlignSide {
+    const uint16_t *top;  // [r][len]: the task update's factor
+    const uint16_t *bot;  // [rc][len]: the centroid's factor
+    int32_t len;
+    int32_t ks;           // K-splits of this side
+};
+struct AlignPairP {
+    AlignSide side[2];    // 0: d_in (A factors), 1: d_out (B factors)
+    int32_t r, rc;
+    float s, s_c;
+};
+struct AlignParams {
+    AlignPairP pair[ALIGN_MAX_PAIRS];
+    int32_t n_pairs;
+    int32_t unit_start[2 * ALIGN_MAX_PAIRS + 1];  // first unit of (pair, side), then the total
+    float *part;                                  // [units][ALIGN_PART]
+    float *loss;
+    float *cosine;                                // may be null
+    float eps;
+    uint32_t *err;                                // set when a bounded wait gave up
+};
+
+__global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_constant__ AlignParams p)
+{
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    uint8_t *ring = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    const uint32_t ring32 = smem_u32(ring);
+    __shared__ uint64_t bar[ALIGN_STAGES];
+    __shared__ uint32_t tmem_slot;
+
+    const int unit = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    int ps = 0;
+    while (ps + 1 < 2 * p.n_pairs && p.unit_start[ps + 1] <= unit) ++ps;
+    const AlignPairP &pr = p.pair[ps >> 1];
+    const AlignSide &sd = pr.side[ps & 1];
+    const int split = unit - p.unit_start[ps];
+    const int r = pr.r, S = pr.r + pr.rc, n_pad = (S + 15) & ~15, len = sd.len;
+    const int nk = (len + 63) / 64;
+    const int c0 = (int)((int64_t)nk * split / sd.ks), n_my = (int)((int64_t)nk * (split + 1) / sd.ks) - c0;
+
+    if (warp == 0) {
+        tmem_alloc(smem_u32(&tmem_slot), 128);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        for (int i = 0; i < ALIGN_STAGES; ++i) mbar_init(smem_u32(&bar[i]), 1);
+        mbar_fence_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    // chunk i of this unit into stage st: rows < S, 16-byte pieces (columns
+    // past len zero-filled); rows >= S are never loaded and only reach
+    // accumulator rows and columns >= S, which are not read
+    auto load = [&](int i, int st) {
+        const int k0 = (c0 + i) * 64;
+        const uint32_t dst = ring32 + st * ALIGN_STAGE_BYTES;
+        for (int idx = tid; idx < S * 8; idx += ALIGN_THREADS) {
+            const int row = idx >> 3, c = idx & 7, col = k0 + c * 8;
+            const uint16_t *src = row < r ? sd.top + (int64_t)row * len : sd.bot + (int64_t)(row - r) * len;
+            const bool ok = col < len;
+            cp_async16(dst + swz128(row, c), ok ? src + col : src, ok);
+        }
+    };
+    const uint32_t idesc = idesc_bf16_f32(128, n_pad);
+    bool ok_all = true;
+    uint32_t phase = 0, pending = 0;
+    for (int st = 0; st < ALIGN_STAGES - 1; ++st) {
+        if (st < n_my) load(st, st);
+        cp_async_commit();
+    }
+    for (int it = 0; it < n_my; ++it) {
+        const int st = it % ALIGN_STAGES;
+        cp_async_wait_dyn(ALIGN_STAGES - 2);
+        fence_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t a = ring32 + st * ALIGN_STAGE_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+                umma_bf16(tmem, sdesc_kmajor_sw128(a + kk * 32), sdesc_kmajor_sw128(a + kk * 32), idesc,
+                          (it > 0 || kk > 0) ? 1u : 0u);
+            umma_commit(smem_u32(&bar[st]));
+        }
+        pending |= 1u << st;
+        const int nxt = it + ALIGN_STAGES - 1;
+        if (nxt < n_my) {
+            // the stage of chunk nxt last held chunk it - 1: its MMAs must be done
+            if (it >= 1) {
+                const int pst = (it - 1) % ALIGN_STAGES;
+                if (!mbar_wait(smem_u32(&bar[pst]), (phase >> pst) & 1)) ok_all = false;
+                phase ^= 1u << pst;
+                pending &= ~(1u << pst);
+            }
+            load(nxt, nxt % ALIGN_STAGES);
+        }
+        cp_async_commit();
+    }
+    cp_async_wait<0>();
+    for (int st = 0; st < ALIGN_STAGES; ++st)
+        if ((pending >> st) & 1) {
+            if (!mbar_wait(smem_u32(&bar[st]), (phase >> st) & 1)) ok_all = false;
+            phase ^= 1u << st;
+        }
+    tc_fence_after();
+
+    // D rows (tensor-memory lanes) = stack rows, columns = stack rows
+    float *out = p.part + (int64_t)unit * ALIGN_PART;
+    const int row = warp * 32 + lane;
+    for (int g = 0; g < n_pad / 16; ++g) {
+        uint32_t v[16];
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + g * 16, v);
+        tmem_ld_wait();
+        if (row < S) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+                if (g * 16 + e < S) out[row * S + g * 16 + e] = __uint_as_float(v[e]);
+        }
+    }
+    if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
+__device__ double block_sum(double v, double *red)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    double t = 0.0;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    __syncthreads();
+    return t;  // valid in thread 0
+}
+
+__global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __grid_constant__ AlignParams p)
+{
+    __shared__ double red[COMBINE_THREADS / 32];
+    const int pi = blockIdx.x;
+    const AlignPairP &pr = p.pair[pi];
+    const int r = pr.r, S = pr.r + pr.rc;
+    const int u_in = p.unit_start[2 * pi], u_out = p.unit_start[2 * pi + 1];
+    const int ks_in = pr.side[0].ks, ks_out = pr.side[1].ks;
+    double num = 0.0, na = 0.0, nc = 0.0;
+    for (int idx = threadIdx.x; idx < S * S; idx += COMBINE_THREADS) {
+        const int i = idx / S, j = idx - i * S;
+        if (i >= r && j < r) continue;  // the lower cross block mirrors the upper one
+        float gi = 0.f, go = 0.f;
+        for (int s = 0; s < ks_in; ++s) gi += p.part[(int64_t)(u_in + s) * ALIGN_PART + idx];
+        for (int s = 0; s < ks_out; ++s) go += p.part[(int64_t)(u_out + s) * ALIGN_PART + idx];
+        const double prod = (double)gi * (double)go;
+        if (i < r && j < r) na += prod;
+        else if (i >= r) nc += prod;
+        else num += prod;
+    }
+    num = block_sum(num, red);
+    na = block_sum(na, red);
+    nc = block_sum(nc, red);
+    if (threadIdx.x == 0) {
+        const double tr = (double)pr.s * (double)pr.s_c * num;
+        const double n_dw = fabs((double)pr.s) * sqrt(fmax(na, 0.0));
+        const double n_wb = fabs((double)pr.s_c) * sqrt(fmax(nc, 0.0));
+        double cosv = tr / (n_dw * n_wb + (double)p.eps);
+        if (*reinterpret_cast<volatile uint32_t *>(p.err) != 0u) cosv = __longlong_as_double(0x7ff8000000000000ll);
+        p.loss[pi] = (float)(1.0 - cosv);
+        if (p.cosine) p.cosine[pi] = (float)cosv;
+    }
+}
+
+bool aligned16(const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; }
+
+}  // namespace
+
+salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
+                           cudaStream_t stream)
+{
+    if (n < 0 || (n > 0 && (!pairs || !loss))) return SALT_ERR_INVALID_ARG;
+    for (int i = 0; i < n; ++i) {
+        const salt_align_pair &q = pairs[i];
+        if (!q.At || !q.B || !q.At_c || !q.B_c) return SALT_ERR_INVALID_ARG;
+        if (q.r < 1 || q.rc < 1 || q.r + q.rc > SALT_MAX_ALIGN_RANK) return SALT_ERR_RANK;
+        if (q.d_in <= 0 || q.d_out <= 0 || (q.d_in % 8) || (q.d_out % 8)) return SALT_ERR_INVALID_ARG;
+        if (!aligned16(q.At) || !aligned16(q.B) || !aligned16(q.At_c) || !aligned16(q.B_c)) return SALT_ERR_ALIGN;
+    }
+    if (n == 0) return SALT_OK;
+    int dev = 0, n_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return SALT_ERR_CUDA;
+    }
+    static unsigned long long configured = 0;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(configured & bit)) {
+        if (cudaFuncSetAttribute(align_gram_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, ALIGN_SMEM) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            return SALT_ERR_CUDA;
+        }
+        configured |= bit;
+    }
+    for (int first = 0; first < n; first += ALIGN_MAX_PAIRS) {
+        const int m = std::min(ALIGN_MAX_PAIRS, n - first);
+        AlignParams p;
+        std::memset(&p, 0, sizeof p);
+        p.n_pairs = m;
+        p.eps = eps;
+        p.loss = loss + first;
+        p.cosine = cosine ? cosine + first : nullptr;
+        // K-splits: at most 64 chunks (4096 columns) a unit, then more
+        // splits while the launch has fewer than three units per SM
+        int nk[2 * ALIGN_MAX_PAIRS], ks[2 * ALIGN_MAX_PAIRS];
+        int64_t units = 0;
+        for (int i = 0; i < m; ++i) {
+            const salt_align_pair &q = pairs[first + i];
+            nk[2 * i] = (q.d_in + 63) / 64;
+            nk[2 * i + 1] = (q.d_out + 63) / 64;
+            for (int sd = 0; sd < 2; ++sd) {
+                ks[2 * i + sd] = (nk[2 * i + sd] + 63) / 64;
+                units += ks[2 * i + sd];
+            }
+        }
+        const int64_t target = 3LL * n_sm;
+        if (units < target) {
+            const int64_t f = (target + units - 1) / units;
+            units = 0;
+            for (int k = 0; k < 2 * m; ++k) {
+                ks[k] = (int)std::min<int64_t>(nk[k], std::min<int64_t>(16, (int64_t)ks[k] * f));
+                units += ks[k];
+            }
+        }
+        int u = 0;
+        for (int i = 0; i < m; ++i) {
+            const salt_align_pair &q = pairs[first + i];
+            AlignPairP &d = p.pair[i];
+            d.r = q.r;
+            d.rc = q.rc;
+            d.s = q.s;
+            d.s_c = q.s_c;
+            d.side[0] = AlignSide{static_cast<const uint16_t *>(q.At), static_cast<const uint16_t *>(q.At_c), q.d_in,
+                                  ks[2 * i]};
+            d.side[1] = AlignSide{static_cast<const uint16_t *>(q.B), static_cast<const uint16_t *>(q.B_c), q.d_out,
+                                  ks[2 * i + 1]};
+            p.unit_start[2 * i] = u;
+            u += ks[2 * i];
+            p.unit_start[2 * i + 1] = u;
+            u += ks[2 * i + 1];
+        }
+        p.unit_start[2 * m] = u;
+        // scratch: the error word, then the partials
+        void *ws = nullptr;
+        const size_t bytes = 256 + (size_t)u * ALIGN_PART * sizeof(float);
+        if (cudaMallocAsync(&ws, bytes, stream) != cudaSuccess) {
+            cudaGetLastError();
+            return SALT_ERR_OOM;
+        }
+        p.err = static_cast<uint32_t *>(ws);
+        p.part = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + 256);
+        cudaError_t e = cudaMemsetAsync(ws, 0, 256, stream);
+        if (e == cudaSuccess) {
+            align_gram_kernel<<<u, ALIGN_THREADS, ALIGN_SMEM, stream>>>(p);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess) {
+            align_combine_kernel<<<m, COMBINE_THREADS, 0, stream>>>(p);
+            e = cudaGetLastError();
+        }
+        cudaError_t f = cudaFreeAsync(ws, stream);
+        if (e != cudaSuccess || f != cudaSuccess) {
+            cudaGetLastError();
+            return SALT_ERR_CUDA;
+        }
+    }
+    return SALT_OK;
+}
+
+}  // namespace salt

@@ -44,6 +44,7 @@
 
 #include <mutex>
 
+#include "salt_async.cuh"
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
 
@@ -87,32 +88,6 @@ struct FusedInfo {
 };
 constexpr size_t FUSED_SMEM = 1024 + RING_BYTES + (sizeof(FusedInfo) + 127) / 128 * 128;
 static_assert(FUSED_SMEM <= 227 * 1024, "shared memory exceeds the per-block limit");
-
-__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ int swz128(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid)
-{
-    int n = valid ? 16 : 0;  // 0: zero-fill, nothing read
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(n));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-// wait until at most n groups are pending (n in [0, 7])
-__device__ __forceinline__ void cp_async_wait_dyn(int n)
-{
-    switch (n) {
-    case 0: cp_async_wait<0>(); break;
-    case 1: cp_async_wait<1>(); break;
-    case 2: cp_async_wait<2>(); break;
-    case 3: cp_async_wait<3>(); break;
-    case 4: cp_async_wait<4>(); break;
-    case 5: cp_async_wait<5>(); break;
-    case 6: cp_async_wait<6>(); break;
-    default: cp_async_wait<7>(); break;
-    }
-}
 
 // arrive on the mbarrier once all of this thread's earlier cp.async copies have landed
 __device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar)
@@ -174,27 +149,10 @@ __device__ bool wait_count(const uint32_t *c, uint32_t n)
     return false;
 }
 
-__device__ __forceinline__ float bf16_to_f(uint16_t h) { return __uint_as_float(((uint32_t)h) << 16); }
-__device__ __forceinline__ uint16_t f_to_bf16(float f)
-{
-    __nv_bfloat16 b = __float2bfloat16_rn(f);
-    return *reinterpret_cast<uint16_t *>(&b);
-}
-
-// Two bf16 (low half first) plus two fp32 deltas, each sum rounded once to
-// bf16 (round to nearest even), packed the same way.
-__device__ __forceinline__ uint32_t add_bf16x2(uint32_t y2, float d_lo, float d_hi)
-{
-    const float lo = __uint_as_float(y2 << 16) + d_lo;
-    const float hi = __uint_as_float(y2 & 0xffff0000u) + d_hi;
-    const __nv_bfloat162 r = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t *>(&r);
-}
-
 // Residual row entry of a block's factor stack -> first element of that row.
 __device__ __forceinline__ const uint16_t *residual_row(const ApplyParams &p, const ApplyProj &pr, int e, bool b_side)
 {
-    const int slot = e >> 8, rank = ((e >> 4) & 15) + 1, k = e & 15;
+    const int slot = res_slot(e), rank = res_rank(e), k = res_k(e);
     const uint16_t *base = reinterpret_cast<const uint16_t *>(p.pool + (int64_t)slot * p.slot_stride +
                                                               SALT_BLOB_HEADER_BYTES) + (int64_t)rank * pr.res_off;
     return b_side ? base + (int64_t)rank * pr.d_in + (int64_t)k * pr.d_out : base + (int64_t)k * pr.d_in;

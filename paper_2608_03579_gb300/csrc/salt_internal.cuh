@@ -37,13 +37,15 @@ __host__ __device__ constexpr int blk_weight(int M, int S) { return 2 * M + S + 
 
 // Device arrays of one segments object.
 struct SegDev {
-    int32_t *ids;          // [2 * max_tokens]: domain ids, then slot ids
+    int32_t *ids;          // [3 * max_tokens]: domain ids, slot ids, then gamma bins
     int32_t *perm;         // [max_tokens] token index in grouped order
     int32_t *sorted_slot;  // [max_tokens] validated slot of the i-th grouped token (-1: none)
-    int32_t *dseg_ptr;     // [max_tokens + 1]
+    int32_t *dseg_ptr;     // [max_tokens + 1] runs of equal (domain, gamma bin)
     int32_t *dseg_dom;     // [max_tokens]
-    int32_t *useg_ptr;     // [max_tokens + 1]
+    int32_t *dseg_gbin;    // [max_tokens]
+    int32_t *useg_ptr;     // [max_tokens + 1] runs of equal (domain, gamma bin, slot)
     int32_t *useg_dom;     // [max_tokens]
+    int32_t *useg_gbin;    // [max_tokens]
     int32_t *useg_slot;    // [max_tokens]
     int32_t *blk;          // [BLK_INTS * max_tokens], see BLK_* below
     int32_t *counts;       // [4]: n_tokens, domain runs, user runs, row blocks
@@ -52,10 +54,17 @@ struct SegDev {
     int32_t *tok_uoff;     // [max_tokens]
     int32_t *tok_urank;    // [max_tokens]
     float *tok_su;         // [max_tokens]
-    // per row block: residual rows of the factor stack,
-    // (slot << 8) | ((rank - 1) << 4) | k
+    // per row block: residual rows of the factor stack, res_code(slot, rank, k)
     int32_t *blk_res;      // [max_tokens * S_MAX]
 };
+
+// Code of one residual row of a factor stack: row k of the rank-`rank`
+// residual in slot `slot` (slot < 2^17, 1 <= rank <= 128, k < rank).
+__host__ __device__ constexpr int32_t res_code(int slot, int rank, int k) { return (slot << 14) | ((rank - 1) << 7) | k; }
+__host__ __device__ constexpr int res_slot(int32_t e) { return e >> 14; }
+__host__ __device__ constexpr int res_rank(int32_t e) { return ((e >> 7) & 127) + 1; }
+__host__ __device__ constexpr int res_k(int32_t e) { return e & 127; }
+static_assert(SALT_MAX_RESIDUAL_RANK <= 128, "a residual row code holds ranks up to 128");
 
 // Scratch of the apply path, owned by a segments object (one apply at a
 // time uses it; applies on different streams are serialised).
@@ -81,7 +90,8 @@ struct ApplyWork {
     uint32_t *vdone;       // [2 * SALT_MAX_GROUP * blk_cap]
     uint32_t *seq;         // [2]
 };
-constexpr int PART_COLS = SALT_MAX_CENTROID_RANK + SALT_MAX_RESIDUAL_RANK;  // centroid | own residual
+constexpr int PART_COLS = SALT_MAX_TOKEN_RANK;  // centroid | own residual, per token
+static_assert(PART_COLS % 4 == 0, "partial rows are read as float4");
 constexpr int PART_CAP = 512;  // partial tiles per segments object (20 MiB)
 
 struct SegParams {
@@ -94,6 +104,9 @@ struct SegParams {
     int32_t umax;
     const int32_t *dom_rc;   // [n_domains] pinned rank, 0 = not pinned
     const float *dom_sc;     // [n_domains] centroid scale
+    int32_t has_gbin;        // ids hold gamma bins
+    int32_t n_gamma;         // gamma bins of this build
+    float gamma[SALT_MAX_GAMMA_BINS];
     const uint8_t *pool;     // slot pool base
     int64_t slot_stride;     // bytes per slot
     uint32_t *err;           // device error word
@@ -140,6 +153,14 @@ cudaError_t apply_prepare(int device);
 // the stream (only when that kernel did not write the segment tables).
 cudaError_t launch_apply(const ApplyParams &p, bool pdl, cudaStream_t stream);
 size_t apply_smem_bytes();
+// W[Mdim][Ndim] += scale * P^T Q for P = [rc][Mdim], Q = [rc][Ndim] (bf16,
+// rows contiguous, rc <= 64): the centroid fold; a timed-out wait sets
+// SALT_DEVERR_TIMEOUT in *err.
+cudaError_t launch_fold(const uint16_t *P, const uint16_t *Q, uint16_t *W, int Mdim, int Ndim, int rc, float scale,
+                        uint32_t *err, cudaStream_t stream);
+// salt_align_loss on the current device.
+salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
+                           cudaStream_t stream);
 // One thread waits, with the apply's bounded cross-CTA wait, on a device word
 // nothing sets; raises SALT_DEVERR_TIMEOUT in *err when it gives up.
 cudaError_t launch_wait_selftest(uint32_t *err, cudaStream_t stream);

@@ -119,11 +119,12 @@ salt_status check_config(const salt_config *c)
         if (c->d_in[l] <= 0 || c->d_out[l] <= 0 || (c->d_in[l] % 8) || (c->d_out[l] % 8))
             return SALT_ERR_INVALID_ARG;
     }
-    if (c->n_domains < 0 || c->n_domains >= (1 << 21)) return SALT_ERR_INVALID_ARG;
-    if (c->n_slots < 0 || c->n_slots >= (1 << 21) - 1) return SALT_ERR_INVALID_ARG;
+    // the segment key holds domain + 1 in 17 bits; a residual row code holds the slot in 17
+    if (c->n_domains < 0 || c->n_domains >= (1 << 17) - 1) return SALT_ERR_INVALID_ARG;
+    if (c->n_slots < 0 || c->n_slots >= (1 << 17)) return SALT_ERR_INVALID_ARG;
     if (c->rc_max < 0 || c->rc_max > SALT_MAX_CENTROID_RANK) return SALT_ERR_RANK;
     if (c->r_max < 1 || c->r_max > SALT_MAX_RESIDUAL_RANK) return SALT_ERR_RANK;
-    if (c->rc_max + c->r_max > S_MAX) return SALT_ERR_RANK;
+    if (c->rc_max + c->r_max > SALT_MAX_TOKEN_RANK) return SALT_ERR_RANK;
     if (c->max_tokens < 1 || c->max_tokens > SALT_MAX_TOKENS) return SALT_ERR_TOO_MANY_TOKENS;
     return SALT_OK;
 }
@@ -160,25 +161,29 @@ void add_stream(std::vector<cudaStream_t> &v, cudaStream_t s)
     v.push_back(s);
 }
 
-// Row blocks of a T-token batch, whatever the ids: blocks <= T/TM + groups
-// and groups <= user runs / umax + domain runs (+ 1 for the skipped run).
-int block_bound_loose(const salt_ctx *ctx, int T)
+// Row blocks of a T-token batch with n_gamma gamma bins, whatever the ids:
+// blocks <= T/TM + groups and groups <= user runs / umax + (domain, bin)
+// runs (+ 1 for the skipped run); there are at most
+// n_domains * (n_gamma + 1) + 1 of the latter.
+int block_bound_loose(const salt_ctx *ctx, int T, int n_gamma)
 {
-    int64_t b = (int64_t)T / TM + (int64_t)T / ctx->umax + ctx->n_domains + 3;
+    int64_t b = (int64_t)T / TM + (int64_t)T / ctx->umax + (int64_t)ctx->n_domains * (n_gamma + 1) + 3;
     return (int)(b < T ? (b > 0 ? b : 1) : (T > 0 ? T : 1));
 }
 
-// Tighter bound from validated host ids: a domain with n tokens (those
-// with a term) in u user runs yields at most ceil(n / TM) + ceil(u / umax)
-// blocks.  Only sizes the launch grid; the block list itself comes from the
-// segment kernel, and CTAs past its count exit at once.
-int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *slot, int T)
+// Tighter bound from validated host ids: a (domain, gamma bin) run with n
+// tokens (those with a term) in u user runs yields at most ceil(n / TM) +
+// ceil(u / umax) blocks.  Only sizes the launch grid; the block list itself
+// comes from the segment kernel, and CTAs past its count exit at once.
+int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *gbin, const int32_t *slot, int T,
+                     int n_gamma)
 {
     std::vector<uint64_t> keys;
     keys.reserve(T);
     for (int t = 0; t < T; ++t) {
         if (dom[t] < 0 && slot[t] < 0) continue;
-        keys.push_back(((uint64_t)(uint32_t)(dom[t] + 1) << 32) | (uint32_t)(slot[t] + 1));
+        const uint32_t g = (gbin && dom[t] >= 0) ? (uint32_t)(gbin[t] + 1) : 0u;
+        keys.push_back(((uint64_t)((uint32_t)(dom[t] + 1) * 32u + g) << 32) | (uint32_t)(slot[t] + 1));
     }
     std::sort(keys.begin(), keys.end());
     int64_t bound = 0;
@@ -195,7 +200,7 @@ int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *slo
         }
         bound += (n + TM - 1) / TM + (u + ctx->umax - 1) / ctx->umax;
     }
-    int cap = block_bound_loose(ctx, ctx->max_tokens);
+    int cap = block_bound_loose(ctx, ctx->max_tokens, n_gamma);
     return (int)(bound < cap ? bound : cap);
 }
 
@@ -289,6 +294,7 @@ const char *salt_status_string(salt_status s)
     case SALT_ERR_DOMAIN_RANGE: return "domain id out of range";
     case SALT_ERR_STALE_SEGMENTS: return "segments refer to a slot reloaded after the build";
     case SALT_ERR_NOT_BUILT: return "segments object not built";
+    case SALT_ERR_GAMMA_RANGE: return "gamma bin out of range";
     }
     return "unknown status";
 }
@@ -473,6 +479,104 @@ salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, flo
     return SALT_OK;
 }
 
+salt_status salt_centroid_fold(salt_ctx *ctx, int32_t domain, int32_t layer, float gamma, void *W, int32_t layout,
+                               salt_stream_t stream)
+{
+    if (!ctx) return SALT_ERR_INVALID_ARG;
+    if (domain < 0 || domain >= ctx->n_domains)
+        return fail(ctx, SALT_ERR_DOMAIN_RANGE, "domain %d outside [0, %d)", domain, ctx->n_domains);
+    if (ctx->dom_rc[domain] == 0) return fail(ctx, SALT_ERR_DOMAIN_NOT_PINNED, "domain %d has no pinned centroid", domain);
+    if (layer < 0 || layer >= ctx->n_layers)
+        return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", layer, ctx->n_layers);
+    if (layout != SALT_W_IN_OUT && layout != SALT_W_OUT_IN) return fail(ctx, SALT_ERR_INVALID_ARG, "unknown layout %d", layout);
+    if (!W) return fail(ctx, SALT_ERR_INVALID_ARG, "null weight");
+    if (reinterpret_cast<uintptr_t>(W) & 15u) return fail(ctx, SALT_ERR_ALIGN, "weight not 16-byte aligned");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    const int din = ctx->d_in[layer], dout = ctx->d_out[layer], rc = ctx->dom_rc[domain];
+    const uint16_t *A = ctx->arenaA + ctx->a_off[layer] + (int64_t)domain * ctx->rc_max * din;
+    const uint16_t *B = ctx->arenaB + ctx->b_off[layer] + (int64_t)domain * ctx->rc_max * dout;
+    const float scale = gamma * ctx->dom_sc[domain];
+    uint16_t *w = static_cast<uint16_t *>(W);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (layout == SALT_W_IN_OUT) CUDA_OR_FAIL(ctx, launch_fold(A, B, w, din, dout, rc, scale, ctx->err_dev, st));
+    else CUDA_OR_FAIL(ctx, launch_fold(B, A, w, dout, din, rc, scale, ctx->err_dev, st));
+    return SALT_OK;
+}
+
+salt_status salt_align_loss(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
+                            salt_stream_t stream)
+{
+    return align_loss_run(n, pairs, eps, loss, cosine, static_cast<cudaStream_t>(stream));
+}
+
+// float -> bf16, round to nearest even (NaN kept quiet)
+static uint16_t host_f32_to_bf16(float f)
+{
+    uint32_t u;
+    std::memcpy(&u, &f, sizeof u);
+    if ((u & 0x7fffffffu) > 0x7f800000u) return (uint16_t)((u >> 16) | 0x40u);
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+static float host_bf16_to_f32(uint16_t h)
+{
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    std::memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+salt_status salt_residual_blob_concat(const salt_config *config, int32_t rc, const void *At_c, const void *B_c,
+                                      float s_c, int32_t rank, const void *At_u, const void *B_u, float s_u,
+                                      void *blob, int64_t blob_bytes)
+{
+    if (rc < 1 || rank < 1) return SALT_ERR_RANK;
+    const int32_t R = rc + rank;
+    int64_t need = salt_residual_blob_bytes(config, R);
+    if (need < 0 || !At_c || !B_c || !At_u || !B_u || !blob) return SALT_ERR_INVALID_ARG;
+    if (R > SALT_MAX_RESIDUAL_RANK) return SALT_ERR_RANK;
+    if (blob_bytes < need) return SALT_ERR_INVALID_ARG;
+    const float s = s_u != 0.f ? s_u : 1.f;
+    const float fc = s_c / s, fu = s_u != 0.f ? 1.f : 0.f;
+    salt_blob_header h;
+    std::memset(&h, 0, sizeof h);
+    h.magic = SALT_BLOB_MAGIC;
+    h.version = 1;
+    h.rank = R;
+    h.n_layers = config->n_layers;
+    h.s_u = s;
+    h.payload_bytes = (uint64_t)payload_elems(config, R) * 2;
+    h.layout_hash = fnv1a_layout(config->n_layers, config->d_in, config->d_out);
+    uint8_t *out = static_cast<uint8_t *>(blob);
+    std::memcpy(out, &h, sizeof h);
+    uint16_t *pay = reinterpret_cast<uint16_t *>(out + SALT_BLOB_HEADER_BYTES);
+    const uint16_t *Ac = static_cast<const uint16_t *>(At_c), *Bc = static_cast<const uint16_t *>(B_c);
+    const uint16_t *Au = static_cast<const uint16_t *>(At_u), *Bu = static_cast<const uint16_t *>(B_u);
+    auto scaled = [](const uint16_t *src, int64_t n, float f, uint16_t *dst) {
+        if (f == 1.f) {
+            std::memcpy(dst, src, (size_t)n * 2);
+            return;
+        }
+        for (int64_t i = 0; i < n; ++i) dst[i] = host_f32_to_bf16(f * host_bf16_to_f32(src[i]));
+    };
+    int64_t oc_a = 0, oc_b = 0, ou_a = 0, ou_b = 0, op = 0;
+    for (int l = 0; l < config->n_layers; ++l) {
+        const int64_t di = config->d_in[l], dout = config->d_out[l];
+        std::memcpy(pay + op, Ac + oc_a, (size_t)(rc * di) * 2);
+        std::memcpy(pay + op + rc * di, Au + ou_a, (size_t)(rank * di) * 2);
+        op += R * di;
+        scaled(Bc + oc_b, rc * dout, fc, pay + op);
+        scaled(Bu + ou_b, rank * dout, fu, pay + op + rc * dout);
+        op += R * dout;
+        oc_a += rc * di;
+        ou_a += rank * di;
+        oc_b += rc * dout;
+        ou_b += rank * dout;
+    }
+    return SALT_OK;
+}
+
 salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob, salt_stream_t side_stream)
 {
     if (!ctx) return SALT_ERR_INVALID_ARG;
@@ -521,13 +625,14 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
     seg->ctx = ctx;
     const int n = ctx->max_tokens;
     auto alloc = [&](int32_t **p, size_t count) { return cudaMalloc(p, count * sizeof(int32_t)) == cudaSuccess; };
-    bool ok = alloc(&seg->d.ids, 2 * (size_t)n) && alloc(&seg->d.perm, n) && alloc(&seg->d.sorted_slot, n) &&
-              alloc(&seg->d.dseg_ptr, n + 1) && alloc(&seg->d.dseg_dom, n) && alloc(&seg->d.useg_ptr, n + 1) &&
-              alloc(&seg->d.useg_dom, n) && alloc(&seg->d.useg_slot, n) &&
+    bool ok = alloc(&seg->d.ids, 3 * (size_t)n) && alloc(&seg->d.perm, n) && alloc(&seg->d.sorted_slot, n) &&
+              alloc(&seg->d.dseg_ptr, n + 1) && alloc(&seg->d.dseg_dom, n) && alloc(&seg->d.dseg_gbin, n) &&
+              alloc(&seg->d.useg_ptr, n + 1) && alloc(&seg->d.useg_dom, n) && alloc(&seg->d.useg_gbin, n) &&
+              alloc(&seg->d.useg_slot, n) &&
               alloc(&seg->d.blk, (size_t)BLK_INTS * n) && alloc(&seg->d.counts, 4) && alloc(&seg->d.tok_uoff, n) &&
               alloc(&seg->d.tok_urank, n) && alloc(reinterpret_cast<int32_t **>(&seg->d.tok_su), n) &&
               alloc(&seg->d.blk_res, (size_t)n * S_MAX);
-    seg->work.blk_cap = block_bound_loose(ctx, n);
+    seg->work.blk_cap = block_bound_loose(ctx, n, SALT_MAX_GAMMA_BINS);
     seg->work.part_cap = PART_CAP;
     const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
     ok = ok && cudaMalloc(&seg->work.vext, n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
@@ -540,7 +645,7 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
          cudaMemset(seg->work.seq, 0, 2 * sizeof(uint32_t)) == cudaSuccess &&
          apply_encode_vmap(seg->work) == cudaSuccess;
     for (int i = 0; ok && i < 2; ++i) {
-        ok = cudaHostAlloc(&seg->staging[i], 2 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
+        ok = cudaHostAlloc(&seg->staging[i], 3 * (size_t)n * sizeof(int32_t), cudaHostAllocDefault) == cudaSuccess &&
              cudaEventCreateWithFlags(&seg->staging_ev[i], cudaEventDisableTiming) == cudaSuccess;
     }
     ok = ok && cudaEventCreateWithFlags(&seg->built_ev, cudaEventDisableTiming) == cudaSuccess &&
@@ -567,7 +672,8 @@ void salt_segments_destroy(salt_segments *seg)
     for (int i = 0; i < 2; ++i)
         if (seg->staging_ev[i]) cudaEventSynchronize(seg->staging_ev[i]);
     int32_t *arrs[] = {seg->d.ids, seg->d.perm, seg->d.sorted_slot, seg->d.dseg_ptr, seg->d.dseg_dom,
-                       seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_slot, seg->d.blk, seg->d.counts,
+                       seg->d.dseg_gbin, seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_gbin,
+                       seg->d.useg_slot, seg->d.blk, seg->d.counts,
                        seg->d.tok_uoff, seg->d.tok_urank, reinterpret_cast<int32_t *>(seg->d.tok_su),
                        seg->d.blk_res};
     for (int32_t *p : arrs) cudaFree(p);
@@ -588,19 +694,30 @@ void salt_segments_destroy(salt_segments *seg)
 }
 
 salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t *domain_ids,
-                                const int32_t *slot_ids, int32_t n_tokens, salt_stream_t stream_)
+                                const int32_t *slot_ids, int32_t n_tokens, salt_stream_t stream)
+{
+    return salt_build_segments_gamma(ctx, seg, domain_ids, nullptr, slot_ids, n_tokens, 0, nullptr, stream);
+}
+
+salt_status salt_build_segments_gamma(salt_ctx *ctx, salt_segments *seg, const int32_t *domain_ids,
+                                      const int32_t *gamma_bins, const int32_t *slot_ids, int32_t n_tokens,
+                                      int32_t n_gamma, const float *gamma, salt_stream_t stream_)
 {
     if (!ctx || !seg || seg->ctx != ctx) return SALT_ERR_INVALID_ARG;
     if (n_tokens < 0) return fail(ctx, SALT_ERR_INVALID_ARG, "negative token count");
     if (n_tokens > ctx->max_tokens)
         return fail(ctx, SALT_ERR_TOO_MANY_TOKENS, "%d tokens > max_tokens %d", n_tokens, ctx->max_tokens);
     if (n_tokens > 0 && (!domain_ids || !slot_ids)) return fail(ctx, SALT_ERR_INVALID_ARG, "null id array");
+    if (n_gamma < 0 || n_gamma > SALT_MAX_GAMMA_BINS)
+        return fail(ctx, SALT_ERR_INVALID_ARG, "%d gamma bins outside [0, %d]", n_gamma, SALT_MAX_GAMMA_BINS);
+    if (n_gamma > 0 && !gamma) return fail(ctx, SALT_ERR_INVALID_ARG, "null gamma table");
     if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
     const int T = n_tokens;
+    const bool has_gbin = gamma_bins != nullptr;
     bool dev_ids = T > 0 && is_device_pointer(domain_ids);
-    if (T > 0 && dev_ids != is_device_pointer(slot_ids))
-        return fail(ctx, SALT_ERR_INVALID_ARG, "domain and slot ids must both be host or both be device memory");
+    if (T > 0 && (dev_ids != is_device_pointer(slot_ids) || (has_gbin && dev_ids != is_device_pointer(gamma_bins))))
+        return fail(ctx, SALT_ERR_INVALID_ARG, "the id arrays must all be host or all be device memory");
 
     std::vector<uint8_t> refs;
     if (!dev_ids) {
@@ -618,6 +735,9 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
                     return fail(ctx, SALT_ERR_SLOT_EMPTY, "token %d: slot %d was never loaded", t, s);
                 refs[s] = 1;
             }
+            if (has_gbin && d >= 0 && (gamma_bins[t] < -1 || gamma_bins[t] >= n_gamma))
+                return fail(ctx, SALT_ERR_GAMMA_RANGE, "token %d: gamma bin %d outside [-1, %d)", t, gamma_bins[t],
+                            n_gamma);
         }
     }
     // The device buffers of seg may still be read by earlier uses on other streams.
@@ -632,20 +752,23 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
         ctx->slot_waited_stream[s] = stream;
     }
     if (T > 0) {
+        const int32_t *src[3] = {domain_ids, slot_ids, gamma_bins};
+        const int n_arr = has_gbin ? 3 : 2;
         if (dev_ids) {
-            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids, domain_ids, (size_t)T * 4, cudaMemcpyDeviceToDevice, stream));
-            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + ctx->max_tokens, slot_ids, (size_t)T * 4,
-                                              cudaMemcpyDeviceToDevice, stream));
+            for (int a = 0; a < n_arr; ++a)
+                CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + (size_t)a * ctx->max_tokens, src[a], (size_t)T * 4,
+                                                  cudaMemcpyDeviceToDevice, stream));
         } else {
             int k = seg->staging_next;
             seg->staging_next ^= 1;
             if (seg->staging_used[k]) CUDA_OR_FAIL(ctx, cudaEventSynchronize(seg->staging_ev[k]));
             int32_t *h = seg->staging[k];
-            std::memcpy(h, domain_ids, (size_t)T * 4);
-            std::memcpy(h + ctx->max_tokens, slot_ids, (size_t)T * 4);
-            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids, h, (size_t)T * 4, cudaMemcpyHostToDevice, stream));
-            CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + ctx->max_tokens, h + ctx->max_tokens, (size_t)T * 4,
-                                              cudaMemcpyHostToDevice, stream));
+            for (int a = 0; a < n_arr; ++a) {
+                std::memcpy(h + (size_t)a * ctx->max_tokens, src[a], (size_t)T * 4);
+                CUDA_OR_FAIL(ctx, cudaMemcpyAsync(seg->d.ids + (size_t)a * ctx->max_tokens,
+                                                  h + (size_t)a * ctx->max_tokens, (size_t)T * 4,
+                                                  cudaMemcpyHostToDevice, stream));
+            }
             CUDA_OR_FAIL(ctx, cudaEventRecord(seg->staging_ev[k], stream));
             seg->staging_used[k] = true;
         }
@@ -660,6 +783,9 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
     p.umax = ctx->umax;
     p.dom_rc = ctx->dom_rc_dev;
     p.dom_sc = ctx->dom_sc_dev;
+    p.has_gbin = has_gbin ? 1 : 0;
+    p.n_gamma = n_gamma;
+    for (int g = 0; g < SALT_MAX_GAMMA_BINS; ++g) p.gamma[g] = g < n_gamma ? gamma[g] : 1.f;
     p.pool = ctx->pool;
     p.slot_stride = ctx->slot_stride;
     p.err = ctx->err_dev;
@@ -674,8 +800,10 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg, const int32_t
     if (dev_ids) std::fill(seg->refs.begin(), seg->refs.end(), 1);
     else seg->refs.swap(refs);
     if (T == 0) seg->n_blk_bound = 0;
-    else if (dev_ids) seg->n_blk_bound = std::min(block_bound_loose(ctx, T), seg->work.blk_cap);
-    else seg->n_blk_bound = std::min(block_bound_host(ctx, domain_ids, slot_ids, T), seg->work.blk_cap);
+    else if (dev_ids) seg->n_blk_bound = std::min(block_bound_loose(ctx, T, has_gbin ? n_gamma : 0), seg->work.blk_cap);
+    else
+        seg->n_blk_bound =
+            std::min(block_bound_host(ctx, domain_ids, gamma_bins, slot_ids, T, n_gamma), seg->work.blk_cap);
     seg->build_stream = stream;
     seg->use_streams.clear();
     seg->use_streams.push_back(stream);
@@ -711,6 +839,22 @@ salt_status salt_segments_export(salt_ctx *ctx, const salt_segments *seg, int32_
             blocks[3 * b + 2] = rec[(size_t)BLK_INTS * b + BLK_DOM];
         }
     }
+    return SALT_OK;
+}
+
+salt_status salt_segments_export_gamma(salt_ctx *ctx, const salt_segments *seg, int32_t *dseg_gbin,
+                                       int32_t *useg_gbin)
+{
+    if (!ctx || !seg || seg->ctx != ctx) return SALT_ERR_INVALID_ARG;
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, cudaEventSynchronize(seg->built_ev));
+    int32_t counts[4];
+    CUDA_OR_FAIL(ctx, cudaMemcpy(counts, seg->d.counts, sizeof counts, cudaMemcpyDeviceToHost));
+    if (dseg_gbin && counts[1] > 0)
+        CUDA_OR_FAIL(ctx, cudaMemcpy(dseg_gbin, seg->d.dseg_gbin, (size_t)counts[1] * 4, cudaMemcpyDeviceToHost));
+    if (useg_gbin && counts[2] > 0)
+        CUDA_OR_FAIL(ctx, cudaMemcpy(useg_gbin, seg->d.useg_gbin, (size_t)counts[2] * 4, cudaMemcpyDeviceToHost));
     return SALT_OK;
 }
 

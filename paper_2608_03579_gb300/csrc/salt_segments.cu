@@ -1,20 +1,22 @@
 // Segment builder: groups a heterogeneous batch for the apply kernel.
 //
-// Section "Multi-Tenant Serving" groups requests by their centroid, and the
-// residuals are batched heterogeneously (SGMV, Section "Multi-Tenant LoRA
-// Serving").  One CTA of 1024 threads:
-//   1. validates every (domain, slot) id into the device error word (an
-//      invalid id is treated as -1, never dereferenced),
-//   2. sorts the keys (domain + 1, slot + 1, token) with a bitonic network in
-//      shared memory; keys are unique, so the order is the stable order of
-//      (domain, slot) with ties in token order and -1 first,
-//   3. writes perm / sorted_slot and the maximal domain and user runs
+// Section "Multi-Tenant Serving" groups requests by their (centroid, gamma)
+// pair, and the residuals are batched heterogeneously (SGMV, Section
+// "Multi-Tenant LoRA Serving").  One CTA of 1024 threads:
+//   1. validates every (domain, gamma bin, slot) id into the device error
+//      word (an invalid id is treated as -1, never dereferenced; a token
+//      without a centroid has no bin),
+//   2. sorts the keys (domain + 1, bin + 1, slot + 1, token) with a bitonic
+//      network in shared memory; keys are unique, so the order is the
+//      stable order of (domain, bin, slot) with ties in token order and -1
+//      first,
+//   3. writes perm / sorted_slot and the maximal (domain, bin) and user runs
 //      (two passes over per-thread chunks with a block-wide scan),
-//   4. cuts row blocks for the apply kernel: within a domain run, user runs
-//      are grouped umax at a time and each group is split evenly into
-//      ceil(len / TM) blocks of at most TM tokens.  The leading (-1, -1) run
-//      (tokens with neither term) gets no block, so those rows are never
-//      touched.
+//   4. cuts row blocks for the apply kernel: within a (domain, bin) run, user
+//      runs are grouped umax at a time and each group is split evenly into
+//      ceil(len / TM) blocks of at most TM tokens; a block's centroid scale
+//      is s_c(domain) * gamma[bin].  The leading (-1, -1) run (tokens with
+//      neither term) gets no block, so those rows are never touched.
 // No global scratch is used: the per-group table lives in the shared memory
 // the keys occupied.
 #include "salt_internal.cuh"
@@ -22,12 +24,19 @@
 namespace salt {
 namespace {
 
+// key = (domain + 1) << 47 | (bin + 1) << 42 | (slot + 1) << 21 | token
 constexpr int KEY_TOK_BITS = 21;
 constexpr int KEY_SLOT_BITS = 21;
+constexpr int KEY_GB_BITS = 5;
+constexpr int KEY_CENT_SHIFT = KEY_TOK_BITS + KEY_SLOT_BITS;
 constexpr uint64_t KEY_TOK_MASK = (1ull << KEY_TOK_BITS) - 1;
 constexpr uint64_t KEY_SLOT_MASK = (1ull << KEY_SLOT_BITS) - 1;
+constexpr uint64_t KEY_GB_MASK = (1ull << KEY_GB_BITS) - 1;
+static_assert(SALT_MAX_GAMMA_BINS + 1 <= (1 << KEY_GB_BITS), "gamma bins must fit the key");
 
-__device__ __forceinline__ int key_dom(uint64_t k) { return (int)(k >> (KEY_TOK_BITS + KEY_SLOT_BITS)) - 1; }
+__device__ __forceinline__ int key_dom(uint64_t k) { return (int)(k >> (KEY_CENT_SHIFT + KEY_GB_BITS)) - 1; }
+__device__ __forceinline__ int key_gb(uint64_t k) { return (int)((k >> KEY_CENT_SHIFT) & KEY_GB_MASK) - 1; }
+__device__ __forceinline__ uint64_t key_cent(uint64_t k) { return k >> KEY_CENT_SHIFT; }
 __device__ __forceinline__ int key_slot(uint64_t k) { return (int)((k >> KEY_TOK_BITS) & KEY_SLOT_MASK) - 1; }
 __device__ __forceinline__ int key_tok(uint64_t k) { return (int)(k & KEY_TOK_MASK); }
 __device__ __forceinline__ uint64_t key_pair(uint64_t k) { return k >> KEY_TOK_BITS; }
@@ -91,17 +100,24 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
 
     // 1. validate and build keys
     uint32_t errbits = 0;
-    const int32_t *dom_ids = p.s.ids, *slot_ids = p.s.ids + p.max_tokens;
+    const int32_t *dom_ids = p.s.ids, *slot_ids = p.s.ids + p.max_tokens, *gb_ids = p.s.ids + 2 * p.max_tokens;
     for (int i = tid; i < P2; i += nth) {
         uint64_t key = ~0ull;
         if (i < T) {
-            int d = dom_ids[i], s = slot_ids[i];
+            int d = dom_ids[i], s = slot_ids[i], gb = -1;
             if (d < -1 || d >= p.n_domains) {
                 errbits |= SALT_DEVERR_DOMAIN_RANGE;
                 d = -1;
             } else if (d >= 0 && p.dom_rc[d] <= 0) {
                 errbits |= SALT_DEVERR_DOMAIN_NOT_PINNED;
                 d = -1;
+            }
+            if (p.has_gbin && d >= 0) {
+                gb = gb_ids[i];
+                if (gb < -1 || gb >= p.n_gamma) {
+                    errbits |= SALT_DEVERR_GAMMA_RANGE;
+                    gb = -1;
+                }
             }
             if (s < -1 || s >= p.n_slots) {
                 errbits |= SALT_DEVERR_SLOT_RANGE;
@@ -118,7 +134,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
                     s = -1;
                 }
             }
-            key = ((uint64_t)(d + 1) << (KEY_TOK_BITS + KEY_SLOT_BITS)) |
+            key = ((uint64_t)(d + 1) << (KEY_CENT_SHIFT + KEY_GB_BITS)) | ((uint64_t)(gb + 1) << KEY_CENT_SHIFT) |
                   ((uint64_t)(s + 1) << KEY_TOK_BITS) | (uint64_t)i;
         }
         keys[i] = key;
@@ -150,7 +166,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     int nd = 0, nu = 0;
     for (int i = lo; i < hi; ++i) {
         uint64_t k = keys[i];
-        bool dh = i == 0 || key_dom(k) != key_dom(keys[i - 1]);
+        bool dh = i == 0 || key_cent(k) != key_cent(keys[i - 1]);
         bool uh = i == 0 || key_pair(k) != key_pair(keys[i - 1]);
         nd += dh;
         nu += uh;
@@ -160,19 +176,21 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     int ou = block_exclusive_scan(nu, &n_useg, warp_sums);
     for (int i = lo; i < hi; ++i) {
         uint64_t k = keys[i];
-        int d = key_dom(k), s = key_slot(k);
+        int d = key_dom(k), gb = key_gb(k), s = key_slot(k);
         p.s.perm[i] = key_tok(k);
         p.s.sorted_slot[i] = s;
-        bool dh = i == 0 || d != key_dom(keys[i - 1]);
+        bool dh = i == 0 || key_cent(k) != key_cent(keys[i - 1]);
         bool uh = i == 0 || key_pair(k) != key_pair(keys[i - 1]);
         if (dh) {
             p.s.dseg_ptr[od] = i;
             p.s.dseg_dom[od] = d;
+            p.s.dseg_gbin[od] = gb;
             ++od;
         }
         if (uh) {
             p.s.useg_ptr[ou] = i;
             p.s.useg_dom[ou] = d;
+            p.s.useg_gbin[ou] = gb;
             p.s.useg_slot[ou] = s;
             ++ou;
         }
@@ -228,7 +246,8 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         int a, len;
         group_range(g, &a, &len);
         int q = (len + TM - 1) / TM;
-        int d = p.s.useg_dom[grp_first[g]];
+        int d = p.s.useg_dom[grp_first[g]], gb = p.s.useg_gbin[grp_first[g]];
+        const float sc = d >= 0 ? p.dom_sc[d] * (gb >= 0 ? p.gamma[gb] : 1.f) : 0.f;
         for (int b = 0; b < q; ++b) {
             int s0 = a + (int)(((int64_t)b * len) / q);
             int s1 = a + (int)(((int64_t)(b + 1) * len) / q);
@@ -237,7 +256,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
             rec[BLK_LEN] = s1 - s0;
             rec[BLK_DOM] = d;
             rec[BLK_RC] = d >= 0 ? p.dom_rc[d] : 0;
-            rec[BLK_SC] = __float_as_int(d >= 0 ? p.dom_sc[d] : 0.f);
+            rec[BLK_SC] = __float_as_int(sc);
             ++ob;
         }
     }
@@ -250,8 +269,8 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     __syncthreads();
 
     // 5. per-block factor stacks: the residual rows of block b are the rows
-    //    of its user runs in order, (slot << 8) | ((rank - 1) << 4) | k; each
-    //    token records where its own user's rows start.  One warp per block.
+    //    of its user runs in order (res_code(slot, rank, k)); each token
+    //    records where its own user's rows start.  One warp per block.
     const int lane = tid & 31, warp = tid >> 5, nwarp = nth >> 5;
     for (int b = warp; b < n_blk; b += nwarp) {
         const int s0 = p.s.blk[BLK_INTS * b + BLK_START], M = p.s.blk[BLK_INTS * b + BLK_LEN];
@@ -286,7 +305,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
                 if (contrib > 0)
                     for (int k = 0; k < rank; ++k)
                         if (off + k < S_MAX)
-                            p.s.blk_res[(int64_t)b * S_MAX + off + k] = (slot << 8) | ((rank - 1) << 4) | k;
+                            p.s.blk_res[(int64_t)b * S_MAX + off + k] = res_code(slot, rank, k);
             }
             carry += total;
         }

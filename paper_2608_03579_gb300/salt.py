@@ -28,11 +28,15 @@ STATUS = {
     4: "SALT_ERR_DOMAIN_NOT_PINNED", 5: "SALT_ERR_SLOT_RANGE", 6: "SALT_ERR_RANK", 7: "SALT_ERR_LAYER_RANGE",
     8: "SALT_ERR_ALIGN", 9: "SALT_ERR_BAD_BLOB", 10: "SALT_ERR_DEVICE_IDS", 11: "SALT_ERR_TIMEOUT",
     12: "SALT_ERR_CUDA", 13: "SALT_ERR_SLOT_EMPTY", 14: "SALT_ERR_TOO_MANY_TOKENS", 15: "SALT_ERR_DOMAIN_RANGE",
-    16: "SALT_ERR_STALE_SEGMENTS", 17: "SALT_ERR_NOT_BUILT",
+    16: "SALT_ERR_STALE_SEGMENTS", 17: "SALT_ERR_NOT_BUILT", 18: "SALT_ERR_GAMMA_RANGE",
 }
 SALT_BLOB_HEADER_BYTES = 256
 SALT_MAX_TOKENS = 16384
 SALT_MAX_GROUP = 8
+SALT_MAX_GAMMA_BINS = 16
+SALT_MAX_RESIDUAL_RANK = 80
+SALT_W_IN_OUT = 0
+SALT_W_OUT_IN = 1
 
 
 class SaltError(RuntimeError):
@@ -47,6 +51,13 @@ class salt_config(ctypes.Structure):
                 ("d_out", ctypes.POINTER(ctypes.c_int32)), ("n_domains", ctypes.c_int32),
                 ("rc_max", ctypes.c_int32), ("n_slots", ctypes.c_int32), ("r_max", ctypes.c_int32),
                 ("max_tokens", ctypes.c_int32), ("device", ctypes.c_int32)]
+
+
+class salt_align_pair(ctypes.Structure):
+    _fields_ = [("At", ctypes.c_void_p), ("B", ctypes.c_void_p), ("At_c", ctypes.c_void_p),
+                ("B_c", ctypes.c_void_p), ("r", ctypes.c_int32), ("rc", ctypes.c_int32),
+                ("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32), ("s", ctypes.c_float),
+                ("s_c", ctypes.c_float)]
 
 
 class salt_ctx_info(ctypes.Structure):
@@ -79,6 +90,12 @@ _SIGS = {
     "salt_selftest_wait_timeout": (ctypes.c_int, [_vp, _vp]),
     "salt_host_alloc": (_vp, [_i64]),
     "salt_host_free": (None, [_vp]),
+    "salt_residual_blob_concat": (ctypes.c_int, [ctypes.POINTER(salt_config), _i32, _vp, _vp, _f32, _i32, _vp, _vp,
+                                                 _f32, _vp, _i64]),
+    "salt_centroid_fold": (ctypes.c_int, [_vp, _i32, _i32, _f32, _vp, _i32, _vp]),
+    "salt_build_segments_gamma": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp]),
+    "salt_segments_export_gamma": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
+    "salt_align_loss": (ctypes.c_int, [_i32, ctypes.POINTER(salt_align_pair), _f32, _vp, _vp, _vp]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -167,6 +184,33 @@ def salt_residual_blob_pack(d_in, d_out, rank: int, s_u: float, At_u, B_u, blob,
                                         _ptr(blob), blob_bytes))
 
 
+def salt_residual_blob_concat(d_in, d_out, rc: int, At_c, B_c, s_c: float, rank: int, At_u, B_u, s_u: float,
+                              blob, blob_bytes: int) -> None:
+    """Blob of rank rc + rank holding the scaled centroid and the residual as
+    one standard adapter (the long-tail form)."""
+    cfg = make_config(d_in, d_out)
+    _check(_lib.salt_residual_blob_concat(ctypes.byref(cfg), rc, _ptr(At_c), _ptr(B_c), float(s_c), rank,
+                                          _ptr(At_u), _ptr(B_u), float(s_u), _ptr(blob), blob_bytes))
+
+
+def salt_centroid_fold(ctx, domain: int, layer: int, gamma: float, W, layout: int = SALT_W_IN_OUT,
+                       stream=None) -> None:
+    """W += gamma * s_c(domain) * A_c B_c in place (W a CUDA bf16 tensor)."""
+    _check(_lib.salt_centroid_fold(ctx, domain, layer, float(gamma), _ptr(W), layout, _stream(stream)), ctx)
+
+
+def salt_align_loss(pairs, eps: float, loss, cosine=None, stream=None) -> None:
+    """pairs: sequence of dicts with At, B, At_c, B_c (CUDA bf16 tensors or
+    device addresses), r, rc, d_in, d_out, s, s_c.  loss / cosine: CUDA
+    float32 tensors of len(pairs) (cosine may be None)."""
+    n = len(pairs)
+    arr = (salt_align_pair * max(1, n))()
+    for i, q in enumerate(pairs):
+        arr[i] = salt_align_pair(_ptr(q["At"]), _ptr(q["B"]), _ptr(q["At_c"]), _ptr(q["B_c"]), int(q["r"]),
+                                 int(q["rc"]), int(q["d_in"]), int(q["d_out"]), float(q["s"]), float(q["s_c"]))
+    _check(_lib.salt_align_loss(n, arr, float(eps), _ptr(loss), _ptr(cosine), _stream(stream)))
+
+
 class HostBuffer:
     """Huge-page-backed page-locked host memory from salt_host_alloc, viewed
     as a uint8 torch tensor (``.tensor``); freed by ``close()`` or on
@@ -227,6 +271,29 @@ def salt_build_segments(ctx, seg, domain_ids, slot_ids, n_tokens: int | None = N
         slot_ids = np.ascontiguousarray(slot_ids, dtype=np.int32)
     n = len(domain_ids) if n_tokens is None else n_tokens
     _check(_lib.salt_build_segments(ctx, seg, _ptr(domain_ids), _ptr(slot_ids), n, _stream(stream)), ctx)
+
+
+def salt_build_segments_gamma(ctx, seg, domain_ids, gamma_bins, slot_ids, gamma, n_tokens: int | None = None,
+                              stream=None) -> None:
+    """salt_build_segments with per-token gamma bins; gamma: the bins' values."""
+    if isinstance(domain_ids, np.ndarray):
+        domain_ids = np.ascontiguousarray(domain_ids, dtype=np.int32)
+        slot_ids = np.ascontiguousarray(slot_ids, dtype=np.int32)
+    if isinstance(gamma_bins, np.ndarray):
+        gamma_bins = np.ascontiguousarray(gamma_bins, dtype=np.int32)
+    g = np.ascontiguousarray(gamma, dtype=np.float32)
+    n = len(domain_ids) if n_tokens is None else n_tokens
+    _check(_lib.salt_build_segments_gamma(ctx, seg, _ptr(domain_ids), _ptr(gamma_bins), _ptr(slot_ids), n,
+                                          len(g), g.ctypes.data if len(g) else None, _stream(stream)), ctx)
+
+
+def salt_segments_export_gamma(ctx, seg, max_tokens: int) -> dict:
+    """The gamma bins of the domain runs and user runs of the last build."""
+    counts = salt_segments_export(ctx, seg, max_tokens)["counts"]
+    dg = np.zeros(max_tokens + 1, dtype=np.int32)
+    ug = np.zeros(max_tokens + 1, dtype=np.int32)
+    _check(_lib.salt_segments_export_gamma(ctx, seg, dg.ctypes.data, ug.ctypes.data), ctx)
+    return {"dseg_gbin": dg[:int(counts[1])], "useg_gbin": ug[:int(counts[2])]}
 
 
 def salt_segments_export(ctx, seg, max_tokens: int) -> dict:

@@ -15,8 +15,9 @@ stand in for the paper's trained adapters and datasets, which are not used):
 * residual At_u ~ N(0, 1/d_in), B_u ~ N(0, 1/r_u)
   (the second argument of N is the variance, so each delta term is O(1))
 * a token's domain is its user's slot mod n_domains
-* s_c = s_u = 1 unless a test overrides them (the paper's gamma bins
-  0.6 / 0.8 / 1.0 are exercised by the tests)
+* s_c = s_u = 1 unless a test overrides them
+* gamma bins: the example bins of Section "Multi-Tenant Serving",
+  0.6 / 0.8 / 1.0, each token's bin uniform over them (or -1, no gamma)
 """
 from __future__ import annotations
 
@@ -379,6 +380,18 @@ def config4(seed: int = 4, step: int = 1, n_layers: int = 32, T: int = 512, rank
                         dom_ids=np.full(T, -1, dtype=np.int32), slot_ids=slot, group=groups)
     return Workload("llama8b_32layer_step", seed, layers, 8, [64] * 8, C4_SLOTS, [2] * C4_SLOTS,
                     dom_ids=dom, slot_ids=slot, group=groups)
+
+
+GAMMA_BINS = (0.6, 0.8, 1.0)
+
+
+def gamma_bin_ids(seed: int, T: int, n_bins: int = len(GAMMA_BINS), p_none: float = 0.0) -> np.ndarray:
+    """Per-token gamma bins, uniform over [0, n_bins); with probability
+    p_none a token gets -1 (no gamma)."""
+    g = np.minimum((uniform(seed, stream_id(K_AUX, 5), T) * n_bins).astype(np.int32), n_bins - 1)
+    if p_none > 0:
+        g[uniform(seed, stream_id(K_AUX, 6), T) < p_none] = -1
+    return g.astype(np.int32)
 
 
 CONFIGS = {0: config0, 1: config1, 2: config2, 3: config3, 4: config4}

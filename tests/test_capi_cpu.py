@@ -71,7 +71,9 @@ def test_blob_pack_layout(salt_lib, wl):
     (dict(d_in=[12], d_out=[8]), "SALT_ERR_INVALID_ARG"),           # not a multiple of 8
     (dict(rc_max=65), "SALT_ERR_RANK"),
     (dict(r_max=0), "SALT_ERR_RANK"),
-    (dict(r_max=17), "SALT_ERR_RANK"),
+    (dict(r_max=81), "SALT_ERR_RANK"),
+    (dict(r_max=65), "SALT_ERR_RANK"),                             # rc_max 16 + 65 > 80
+    (dict(n_slots=1 << 17), "SALT_ERR_INVALID_ARG"),
     (dict(max_tokens=16385), "SALT_ERR_TOO_MANY_TOKENS"),
     (dict(max_tokens=0), "SALT_ERR_TOO_MANY_TOKENS"),
 ])

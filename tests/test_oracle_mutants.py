@@ -36,17 +36,18 @@ MUTANTS = {
                                    "keys[t].g = gbin ? gbin[t] : -1;"),
     "gbin_sorted_after_slot": ("    if (a->g != b->g) return a->g < b->g ? -1 : 1;\n    if (a->u != b->u) return a->u < b->u ? -1 : 1;",
                                "    if (a->u != b->u) return a->u < b->u ? -1 : 1;\n    if (a->g != b->g) return a->g < b->g ? -1 : 1;"),
-    "align_B_rank_ignored": ("a += oracle_bf16_value(At[k * d_in + i]) * oracle_bf16_value(B[k * d_out + j]);",
-                             "a += oracle_bf16_value(At[k * d_in + i]) * oracle_bf16_value(B[j]);"),
-    "align_centroid_scale_dropped": ("wb[j] = s_c * c;", "wb[j] = c;"),
+    "align_B_rank_ignored": ("dw[j] += a * oracle_bf16_value(B[k * d_out + j]);",
+                             "dw[j] += a * oracle_bf16_value(B[j]);"),
+    "align_centroid_scale_dropped": ("wb[j] *= s_c;", "wb[j] *= 1.0;"),
     "align_eps_in_numerator": ("double cosine = tr / (n_dw * n_wb + eps);",
                                "double cosine = (tr + eps) / (n_dw * n_wb + eps);"),
     "align_norm_not_rooted": ("double n_dw = sqrt(nn_dw), n_wb = sqrt(nn_wb);",
                               "double n_dw = nn_dw, n_wb = sqrt(nn_wb);"),
     "fold_layout_ignored": ("int64_t idx = layout ? j * d_in + i : i * d_out + j;", "int64_t idx = i * d_out + j;"),
-    "fold_A_transposed": ("acc += oracle_bf16_value(At_c[k * d_in + i])", "acc += oracle_bf16_value(At_c[i * rc + k])"),
-    "fold_scale_dropped": ("W_out[idx] = oracle_bf16_value(W[idx]) + scale * acc;",
-                           "W_out[idx] = oracle_bf16_value(W[idx]) + acc;"),
+    "fold_A_transposed": ("double a = oracle_bf16_value(At_c[k * d_in + i]);\n            for (int64_t j = 0; j < d_out; ++j) row[j]",
+                          "double a = oracle_bf16_value(At_c[i * rc + k]);\n            for (int64_t j = 0; j < d_out; ++j) row[j]"),
+    "fold_scale_dropped": ("W_out[idx] = oracle_bf16_value(W[idx]) + scale * row[j];",
+                           "W_out[idx] = oracle_bf16_value(W[idx]) + row[j];"),
 }
 
 
