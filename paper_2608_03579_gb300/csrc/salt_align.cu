@@ -16,9 +16,12 @@
 // 64-column chunks of F stream through a cp.async ring into a 128-byte-
 // swizzled K-major tile that is both operands of tcgen05.mma
 // (D[128 x S] += F_chunk F_chunk^T, fp32 in tensor memory); the unit writes
-// its S x S partial.  align_combine_kernel: one CTA per pair sums the
-// partials of each side over the splits in split order (fp32), forms the
-// three block sums of G_in o G_out in fp64 and writes the loss.
+// its S x S partial.  align_combine_kernel: COMBINE_CTAS CTAs per pair, each
+// over a slice of the S x S entries, sum the partials of each side over the
+// splits in split order (fp32) and form the three block sums of
+// G_in o G_out in fp64; the last CTA of a pair to finish (a counter) adds
+// the slices' sums in slice order and writes the loss, so the result does
+// not depend on timing.
 #include "salt_async.cuh"
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
@@ -34,9 +37,11 @@ constexpr int ALIGN_THREADS = 128;
 constexpr int ALIGN_STAGES = 4;
 constexpr int ALIGN_STAGE_BYTES = 128 * 128;     // <= 128 stacked rows x 64 columns
 constexpr int ALIGN_SMEM = 1024 + ALIGN_STAGES * ALIGN_STAGE_BYTES;
-constexpr int ALIGN_MAX_PAIRS = 32;              // pairs per launch
+constexpr int ALIGN_MAX_PAIRS = 256;             // pairs per launch (the parameter block stays < 32 KB)
 constexpr int ALIGN_PART = 128 * 128;            // floats per unit partial (row pitch S)
 constexpr int COMBINE_THREADS = 256;
+constexpr int COMBINE_CTAS = 8;                  // CTAs per pair in the combine
+constexpr int KS_CAP = 16;                       // K-splits of one side at most
 static_assert(SALT_MAX_ALIGN_RANK <= 128, "a stack is the 128-row UMMA operand");
 
 struct AlignSide {
@@ -55,11 +60,14 @@ struct AlignParams {
     int32_t n_pairs;
     int32_t unit_start[2 * ALIGN_MAX_PAIRS + 1];  // first unit of (pair, side), then the total
     float *part;                                  // [units][ALIGN_PART]
+    double *sums;                                 // [pairs][COMBINE_CTAS][3]
+    uint32_t *done;                               // [pairs]: combine CTAs finished (zeroed)
     float *loss;
     float *cosine;                                // may be null
     float eps;
     uint32_t *err;                                // set when a bounded wait gave up
 };
+static_assert(sizeof(AlignParams) <= 32000, "kernel parameter block too large");
 
 __global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_constant__ AlignParams p)
 {
@@ -70,8 +78,13 @@ __global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_
     __shared__ uint32_t tmem_slot;
 
     const int unit = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    int ps = 0;
-    while (ps + 1 < 2 * p.n_pairs && p.unit_start[ps + 1] <= unit) ++ps;
+    // the (pair, side) of this unit: the last ps with unit_start[ps] <= unit
+    int ps = 0, hi = 2 * p.n_pairs;
+    while (hi - ps > 1) {
+        const int mid = (ps + hi) >> 1;
+        if (p.unit_start[mid] <= unit) ps = mid;
+        else hi = mid;
+    }
     const AlignPairP &pr = p.pair[ps >> 1];
     const AlignSide &sd = pr.side[ps & 1];
     const int split = unit - p.unit_start[ps];
@@ -181,21 +194,34 @@ __device__ double block_sum(double v, double *red)
     return t;  // valid in thread 0
 }
 
+// sum over the K-splits of one Gram entry, split order; the loads are issued together
+__device__ __forceinline__ float split_sum(const float *part, int u0, int ks, int idx)
+{
+    float v[KS_CAP];
+#pragma unroll
+    for (int s = 0; s < KS_CAP; ++s) v[s] = s < ks ? __ldcg(part + (int64_t)(u0 + s) * ALIGN_PART + idx) : 0.f;
+    float acc = v[0];
+#pragma unroll
+    for (int s = 1; s < KS_CAP; ++s) acc += v[s];
+    return acc;
+}
+
 __global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __grid_constant__ AlignParams p)
 {
     __shared__ double red[COMBINE_THREADS / 32];
-    const int pi = blockIdx.x;
+    __shared__ bool last;
+    const int pi = blockIdx.x / COMBINE_CTAS, slice = blockIdx.x - pi * COMBINE_CTAS;
     const AlignPairP &pr = p.pair[pi];
     const int r = pr.r, S = pr.r + pr.rc;
     const int u_in = p.unit_start[2 * pi], u_out = p.unit_start[2 * pi + 1];
     const int ks_in = pr.side[0].ks, ks_out = pr.side[1].ks;
+    const int i0 = S * S * slice / COMBINE_CTAS, i1 = S * S * (slice + 1) / COMBINE_CTAS;
     double num = 0.0, na = 0.0, nc = 0.0;
-    for (int idx = threadIdx.x; idx < S * S; idx += COMBINE_THREADS) {
+    for (int idx = i0 + threadIdx.x; idx < i1; idx += COMBINE_THREADS) {
         const int i = idx / S, j = idx - i * S;
         if (i >= r && j < r) continue;  // the lower cross block mirrors the upper one
-        float gi = 0.f, go = 0.f;
-        for (int s = 0; s < ks_in; ++s) gi += p.part[(int64_t)(u_in + s) * ALIGN_PART + idx];
-        for (int s = 0; s < ks_out; ++s) go += p.part[(int64_t)(u_out + s) * ALIGN_PART + idx];
+        const float gi = split_sum(p.part, u_in, ks_in, idx);
+        const float go = split_sum(p.part, u_out, ks_out, idx);
         const double prod = (double)gi * (double)go;
         if (i < r && j < r) na += prod;
         else if (i >= r) nc += prod;
@@ -205,6 +231,23 @@ __global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __
     na = block_sum(na, red);
     nc = block_sum(nc, red);
     if (threadIdx.x == 0) {
+        double *o = p.sums + ((int64_t)pi * COMBINE_CTAS + slice) * 3;
+        o[0] = num;
+        o[1] = na;
+        o[2] = nc;
+        __threadfence();
+        last = atomicAdd(p.done + pi, 1u) == COMBINE_CTAS - 1;
+    }
+    __syncthreads();
+    if (last && threadIdx.x == 0) {
+        __threadfence();
+        num = na = nc = 0.0;
+        for (int c = 0; c < COMBINE_CTAS; ++c) {
+            const volatile double *q = p.sums + ((int64_t)pi * COMBINE_CTAS + c) * 3;
+            num += q[0];
+            na += q[1];
+            nc += q[2];
+        }
         const double tr = (double)pr.s * (double)pr.s_c * num;
         const double n_dw = fabs((double)pr.s) * sqrt(fmax(na, 0.0));
         const double n_wb = fabs((double)pr.s_c) * sqrt(fmax(nc, 0.0));
@@ -256,7 +299,7 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
         p.loss = loss + first;
         p.cosine = cosine ? cosine + first : nullptr;
         // K-splits: at most 64 chunks (4096 columns) a unit, then more
-        // splits while the launch has fewer than three units per SM
+        // splits (up to KS_CAP) while the launch has fewer than three units per SM
         int nk[2 * ALIGN_MAX_PAIRS], ks[2 * ALIGN_MAX_PAIRS];
         int64_t units = 0;
         for (int i = 0; i < m; ++i) {
@@ -264,7 +307,7 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
             nk[2 * i] = (q.d_in + 63) / 64;
             nk[2 * i + 1] = (q.d_out + 63) / 64;
             for (int sd = 0; sd < 2; ++sd) {
-                ks[2 * i + sd] = (nk[2 * i + sd] + 63) / 64;
+                ks[2 * i + sd] = std::min(KS_CAP, (nk[2 * i + sd] + 63) / 64);
                 units += ks[2 * i + sd];
             }
         }
@@ -273,7 +316,7 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
             const int64_t f = (target + units - 1) / units;
             units = 0;
             for (int k = 0; k < 2 * m; ++k) {
-                ks[k] = (int)std::min<int64_t>(nk[k], std::min<int64_t>(16, (int64_t)ks[k] * f));
+                ks[k] = (int)std::min<int64_t>(nk[k], std::min<int64_t>(KS_CAP, (int64_t)ks[k] * f));
                 units += ks[k];
             }
         }
@@ -295,22 +338,28 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
             u += ks[2 * i + 1];
         }
         p.unit_start[2 * m] = u;
-        // scratch: the error word, then the partials
+        // scratch: the error word and the pairs' counters (zeroed), the
+        // combine's slice sums, then the partials
+        const size_t head = 256 + (size_t)ALIGN_MAX_PAIRS * 4;
+        const size_t sums = (size_t)ALIGN_MAX_PAIRS * COMBINE_CTAS * 3 * sizeof(double);
         void *ws = nullptr;
-        const size_t bytes = 256 + (size_t)u * ALIGN_PART * sizeof(float);
+        const size_t bytes = head + sums + (size_t)u * ALIGN_PART * sizeof(float);
         if (cudaMallocAsync(&ws, bytes, stream) != cudaSuccess) {
             cudaGetLastError();
             return SALT_ERR_OOM;
         }
-        p.err = static_cast<uint32_t *>(ws);
-        p.part = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + 256);
-        cudaError_t e = cudaMemsetAsync(ws, 0, 256, stream);
+        uint8_t *w8 = static_cast<uint8_t *>(ws);
+        p.err = reinterpret_cast<uint32_t *>(w8);
+        p.done = reinterpret_cast<uint32_t *>(w8 + 256);
+        p.sums = reinterpret_cast<double *>(w8 + head);
+        p.part = reinterpret_cast<float *>(w8 + head + sums);
+        cudaError_t e = cudaMemsetAsync(ws, 0, head, stream);
         if (e == cudaSuccess) {
             align_gram_kernel<<<u, ALIGN_THREADS, ALIGN_SMEM, stream>>>(p);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) {
-            align_combine_kernel<<<m, COMBINE_THREADS, 0, stream>>>(p);
+            align_combine_kernel<<<m * COMBINE_CTAS, COMBINE_THREADS, 0, stream>>>(p);
             e = cudaGetLastError();
         }
         cudaError_t f = cudaFreeAsync(ws, stream);

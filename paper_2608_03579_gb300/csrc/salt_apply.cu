@@ -20,7 +20,8 @@
 //       fp32 partial, waits (bounded) until all splits of the block have,
 //       and then reduces its own slice of the token rows over the splits in
 //       split order (so the result does not depend on timing), writing
-//           V_ext[t,s] = s_c V[t,s]    for s < rc (centroid rows)
+//           V_ext[t,s] = s_c V[t,s]    for s < rc (centroid rows; s_c is the
+//                                      token's: the domain's scale times its gamma)
 //                      = s_u V[t,s]    for s in the token's own user's rows
 //                      = 0             otherwise
 //       as bf16.  Each unit then counts its rows as written.
@@ -76,6 +77,7 @@ struct FusedInfo {
     int32_t ucol[TM];            // first stacked row of the token's user, -1: none
     int32_t urank[TM];
     float usu[TM];
+    float usc[TM];               // the token's centroid scale
     int16_t rt0[S_MAX];          // residual stack row -> first token of its user run
     int16_t rt1[S_MAX];          //                    -> one past the last token
     int16_t rk[S_MAX];           //                    -> rank index within the user
@@ -283,7 +285,6 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
         const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
         const int S = rc + m1.x;
-        const float s_c = __int_as_float(m1.y);
         const int d_in = pr.d_in;
         const int nk = (d_in + KC - 1) / KC;
         const int c0 = split_lo(nk, s, KS), n_my = split_lo(nk, s + 1, KS) - c0;
@@ -300,6 +301,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             info.ucol[t] = uo >= 0 ? rc + uo : -1;
             info.urank[t] = ur;
             info.usu[t] = p.tok_su[start + t];
+            info.usc[t] = p.tok_sc[start + t];
             if (uo >= 0) {
                 const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
                 const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
@@ -439,7 +441,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                         const int t = g * 16 + e;
                         if (t < M) {
                             float val = 0.f;
-                            if (sr < rc) val = s_c * __uint_as_float(v[e]);
+                            if (sr < rc) val = info.usc[t] * __uint_as_float(v[e]);
                             else if (t >= t0 && t < t1) val = info.usu[t] * __uint_as_float(v[e]);
                             Vs[t * VEXT_COLS + sr] = f_to_bf16(val);
                         }
@@ -527,7 +529,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                     for (int e = 0; e < 2; ++e) {
                         const int c = ch * 8 + 2 * hh + e;
                         float val = 0.f;
-                        if (c < rc) val = s_c * ps[c];
+                        if (c < rc) val = info.usc[t] * ps[c];
                         else if (uc >= 0 && c >= uc && c < uc + ur) val = us * ps[rc + (c - uc)];
                         v2[e] = f_to_bf16(val);
                     }

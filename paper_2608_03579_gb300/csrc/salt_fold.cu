@@ -9,8 +9,8 @@
 // W[d_out][d_in], P = B_c and Q = At_c.  K = rc <= 64: a rank-rc update of a
 // large matrix, bound by reading and writing W once.
 //
-// Items are (128-row tile of W, 64 columns); each CTA takes a contiguous
-// range of them, so it mostly stays on one row tile.  Per row tile the CTA
+// Items are (128-row tile of W, 64 columns); each CTA (two per SM) takes a
+// contiguous range of them, so it mostly stays on one row tile.  Per row tile the CTA
 // transposes P's 128 columns into a K-major 128-byte-swizzled tile (the
 // UMMA A operand, K padded to a multiple of 16 with zeros); per item the Q
 // columns (MN-major, as they lie in memory) and the W tile stream through a
@@ -29,13 +29,14 @@ namespace {
 constexpr int FOLD_THREADS = 256;
 constexpr int FOLD_TM = 128;                          // W rows per tile (UMMA M)
 constexpr int FOLD_NC = 64;                           // W columns per item (UMMA N)
-constexpr int FOLD_STAGES = 6;
+constexpr int FOLD_STAGES = 3;
+constexpr int FOLD_CTAS_PER_SM = 2;                   // one CTA's epilogue overlaps the other's copies
 constexpr int FOLD_Q_BYTES = 64 * 128;                // [K <= 64][64 columns], MN-major
 constexpr int FOLD_W_BYTES = FOLD_TM * 128;           // [128 rows][64 columns], swizzled rows
 constexpr int FOLD_STAGE_BYTES = FOLD_Q_BYTES + FOLD_W_BYTES;
 constexpr int FOLD_A_BYTES = FOLD_TM * 128;           // [128 rows][K <= 64], K-major
 constexpr int FOLD_SMEM = 1024 + 2 * FOLD_A_BYTES + FOLD_STAGES * FOLD_STAGE_BYTES;
-static_assert(FOLD_SMEM <= 227 * 1024, "fold shared memory exceeds the per-block limit");
+static_assert(FOLD_CTAS_PER_SM * (FOLD_SMEM + 1024) <= 228 * 1024, "two fold CTAs must fit one SM");
 static_assert(SALT_MAX_CENTROID_RANK <= 64, "K of the fold is one 128-byte row");
 
 struct FoldParams {
@@ -47,7 +48,7 @@ struct FoldParams {
     uint32_t *err;
 };
 
-__global__ void __launch_bounds__(FOLD_THREADS, 1) salt_fold_kernel(const __grid_constant__ FoldParams p)
+__global__ void __launch_bounds__(FOLD_THREADS, FOLD_CTAS_PER_SM) salt_fold_kernel(const __grid_constant__ FoldParams p)
 {
     extern __shared__ __align__(128) uint8_t smem_raw[];
     uint8_t *base = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
@@ -221,7 +222,8 @@ cudaError_t launch_fold(const uint16_t *P, const uint16_t *Q, uint16_t *W, int M
     }
     FoldParams p{P, Q, W, Mdim, Ndim, rc, scale, err};
     const int64_t items = (int64_t)((Mdim + FOLD_TM - 1) / FOLD_TM) * ((Ndim + FOLD_NC - 1) / FOLD_NC);
-    const int grid = (int)(items < n_sm ? items : n_sm);
+    const int64_t slots = (int64_t)FOLD_CTAS_PER_SM * n_sm;
+    const int grid = (int)(items < slots ? items : slots);
     if (grid <= 0) return cudaSuccess;
     salt_fold_kernel<<<grid, FOLD_THREADS, FOLD_SMEM, stream>>>(p);
     return cudaGetLastError();

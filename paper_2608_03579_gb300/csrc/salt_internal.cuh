@@ -11,7 +11,8 @@
 namespace salt {
 
 // Row blocks handed to the apply kernel hold at most TM tokens of one
-// domain and at most `umax` user runs, chosen so that the concatenated
+// domain (of any gamma bins: gamma scales each token's centroid columns of
+// V) and at most `umax` user runs, chosen so that the concatenated
 // factor stack [A_c | a_u1 | a_u2 | ...] of a block never exceeds S_MAX
 // rows: rc_max + umax * r_max <= S_MAX.
 constexpr int TM = 128;
@@ -54,6 +55,8 @@ struct SegDev {
     int32_t *tok_uoff;     // [max_tokens]
     int32_t *tok_urank;    // [max_tokens]
     float *tok_su;         // [max_tokens]
+    // per grouped token: its centroid scale s_c(domain) * gamma[bin] (0: no centroid)
+    float *tok_sc;         // [max_tokens]
     // per row block: residual rows of the factor stack, res_code(slot, rank, k)
     int32_t *blk_res;      // [max_tokens * S_MAX]
 };
@@ -133,6 +136,7 @@ struct ApplyParams {
     const int32_t *tok_uoff;
     const int32_t *tok_urank;
     const float *tok_su;
+    const float *tok_sc;
     const int32_t *blk_res;
     int32_t rc_max;
     const uint8_t *pool;

@@ -161,29 +161,27 @@ void add_stream(std::vector<cudaStream_t> &v, cudaStream_t s)
     v.push_back(s);
 }
 
-// Row blocks of a T-token batch with n_gamma gamma bins, whatever the ids:
-// blocks <= T/TM + groups and groups <= user runs / umax + (domain, bin)
-// runs (+ 1 for the skipped run); there are at most
-// n_domains * (n_gamma + 1) + 1 of the latter.
-int block_bound_loose(const salt_ctx *ctx, int T, int n_gamma)
+// Row blocks of a T-token batch, whatever the ids: blocks <= T/TM + groups
+// and groups <= user runs / umax + domains (+ 1 for the skipped run).
+int block_bound_loose(const salt_ctx *ctx, int T)
 {
-    int64_t b = (int64_t)T / TM + (int64_t)T / ctx->umax + (int64_t)ctx->n_domains * (n_gamma + 1) + 3;
+    int64_t b = (int64_t)T / TM + (int64_t)T / ctx->umax + ctx->n_domains + 3;
     return (int)(b < T ? (b > 0 ? b : 1) : (T > 0 ? T : 1));
 }
 
-// Tighter bound from validated host ids: a (domain, gamma bin) run with n
-// tokens (those with a term) in u user runs yields at most ceil(n / TM) +
-// ceil(u / umax) blocks.  Only sizes the launch grid; the block list itself
-// comes from the segment kernel, and CTAs past its count exit at once.
-int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *gbin, const int32_t *slot, int T,
-                     int n_gamma)
+// Tighter bound from validated host ids: a domain with n tokens (those
+// with a term) in u user runs (runs of equal gamma bin and slot) yields at
+// most ceil(n / TM) + ceil(u / umax) blocks.  Only sizes the launch grid;
+// the block list itself comes from the segment kernel, and CTAs past its
+// count exit at once.
+int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *gbin, const int32_t *slot, int T)
 {
     std::vector<uint64_t> keys;
     keys.reserve(T);
     for (int t = 0; t < T; ++t) {
         if (dom[t] < 0 && slot[t] < 0) continue;
         const uint32_t g = (gbin && dom[t] >= 0) ? (uint32_t)(gbin[t] + 1) : 0u;
-        keys.push_back(((uint64_t)((uint32_t)(dom[t] + 1) * 32u + g) << 32) | (uint32_t)(slot[t] + 1));
+        keys.push_back(((uint64_t)(uint32_t)(dom[t] + 1) << 32) | (g << 20) | (uint32_t)(slot[t] + 1));
     }
     std::sort(keys.begin(), keys.end());
     int64_t bound = 0;
@@ -200,7 +198,7 @@ int block_bound_host(const salt_ctx *ctx, const int32_t *dom, const int32_t *gbi
         }
         bound += (n + TM - 1) / TM + (u + ctx->umax - 1) / ctx->umax;
     }
-    int cap = block_bound_loose(ctx, ctx->max_tokens, n_gamma);
+    int cap = block_bound_loose(ctx, ctx->max_tokens);
     return (int)(bound < cap ? bound : cap);
 }
 
@@ -631,8 +629,9 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
               alloc(&seg->d.useg_slot, n) &&
               alloc(&seg->d.blk, (size_t)BLK_INTS * n) && alloc(&seg->d.counts, 4) && alloc(&seg->d.tok_uoff, n) &&
               alloc(&seg->d.tok_urank, n) && alloc(reinterpret_cast<int32_t **>(&seg->d.tok_su), n) &&
+              alloc(reinterpret_cast<int32_t **>(&seg->d.tok_sc), n) &&
               alloc(&seg->d.blk_res, (size_t)n * S_MAX);
-    seg->work.blk_cap = block_bound_loose(ctx, n, SALT_MAX_GAMMA_BINS);
+    seg->work.blk_cap = block_bound_loose(ctx, n);
     seg->work.part_cap = PART_CAP;
     const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
     ok = ok && cudaMalloc(&seg->work.vext, n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
@@ -675,6 +674,7 @@ void salt_segments_destroy(salt_segments *seg)
                        seg->d.dseg_gbin, seg->d.useg_ptr, seg->d.useg_dom, seg->d.useg_gbin,
                        seg->d.useg_slot, seg->d.blk, seg->d.counts,
                        seg->d.tok_uoff, seg->d.tok_urank, reinterpret_cast<int32_t *>(seg->d.tok_su),
+                       reinterpret_cast<int32_t *>(seg->d.tok_sc),
                        seg->d.blk_res};
     for (int32_t *p : arrs) cudaFree(p);
     cudaFree(seg->work.vext);
@@ -800,10 +800,8 @@ salt_status salt_build_segments_gamma(salt_ctx *ctx, salt_segments *seg, const i
     if (dev_ids) std::fill(seg->refs.begin(), seg->refs.end(), 1);
     else seg->refs.swap(refs);
     if (T == 0) seg->n_blk_bound = 0;
-    else if (dev_ids) seg->n_blk_bound = std::min(block_bound_loose(ctx, T, has_gbin ? n_gamma : 0), seg->work.blk_cap);
-    else
-        seg->n_blk_bound =
-            std::min(block_bound_host(ctx, domain_ids, gamma_bins, slot_ids, T, n_gamma), seg->work.blk_cap);
+    else if (dev_ids) seg->n_blk_bound = std::min(block_bound_loose(ctx, T), seg->work.blk_cap);
+    else seg->n_blk_bound = std::min(block_bound_host(ctx, domain_ids, gamma_bins, slot_ids, T), seg->work.blk_cap);
     seg->build_stream = stream;
     seg->use_streams.clear();
     seg->use_streams.push_back(stream);
@@ -906,6 +904,7 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
     p.tok_uoff = seg->d.tok_uoff;
     p.tok_urank = seg->d.tok_urank;
     p.tok_su = seg->d.tok_su;
+    p.tok_sc = seg->d.tok_sc;
     p.blk_res = seg->d.blk_res;
     p.rc_max = ctx->rc_max;
     p.pool = ctx->pool;
@@ -973,6 +972,7 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     p.tok_uoff = seg->d.tok_uoff;
     p.tok_urank = seg->d.tok_urank;
     p.tok_su = seg->d.tok_su;
+    p.tok_sc = seg->d.tok_sc;
     p.blk_res = seg->d.blk_res;
     p.rc_max = ctx->rc_max;
     p.pool = ctx->pool;

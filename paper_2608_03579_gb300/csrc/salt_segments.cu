@@ -12,11 +12,13 @@
 //      first,
 //   3. writes perm / sorted_slot and the maximal (domain, bin) and user runs
 //      (two passes over per-thread chunks with a block-wide scan),
-//   4. cuts row blocks for the apply kernel: within a (domain, bin) run, user
-//      runs are grouped umax at a time and each group is split evenly into
-//      ceil(len / TM) blocks of at most TM tokens; a block's centroid scale
-//      is s_c(domain) * gamma[bin].  The leading (-1, -1) run (tokens with
-//      neither term) gets no block, so those rows are never touched.
+//   4. cuts row blocks for the apply kernel: within a domain (over all of
+//      its bins), user runs are grouped umax at a time and each group is
+//      split evenly into ceil(len / TM) blocks of at most TM tokens.  gamma
+//      enters as each token's centroid scale s_c(domain) * gamma[bin], so the
+//      bins of one centroid share its blocks and factor reads.  The leading
+//      (-1, -1) run (tokens with neither term) gets no block, so those rows
+//      are never touched.
 // No global scratch is used: the per-group table lives in the shared memory
 // the keys occupied.
 #include "salt_internal.cuh"
@@ -179,6 +181,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         int d = key_dom(k), gb = key_gb(k), s = key_slot(k);
         p.s.perm[i] = key_tok(k);
         p.s.sorted_slot[i] = s;
+        p.s.tok_sc[i] = d >= 0 ? p.dom_sc[d] * (gb >= 0 ? p.gamma[gb] : 1.f) : 0.f;
         bool dh = i == 0 || key_cent(k) != key_cent(keys[i - 1]);
         bool uh = i == 0 || key_pair(k) != key_pair(keys[i - 1]);
         if (dh) {
@@ -202,7 +205,8 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     const bool skip0 = key_dom(keys[0]) == -1 && key_slot(keys[0]) == -1;
     __syncthreads();  // keys are dead from here; run arrays are visible block-wide
 
-    // 4a. group heads over user runs
+    // 4a. group heads over user runs; a group stays within one domain (the
+    //     (domain, bin) runs of a domain are consecutive)
     int32_t *grp_first = reinterpret_cast<int32_t *>(keys);  // [n_groups]
     const int Eu = (n_useg + nth - 1) / nth;
     const int ulo = min(n_useg, tid * Eu), uhi = min(n_useg, ulo + Eu);
@@ -211,8 +215,10 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         if (skip0 && j == 1) return true;
         int start = p.s.useg_ptr[j];
         int dr = upper_index(p.s.dseg_ptr, 0, n_dseg, start);
+        const int d = p.s.dseg_dom[dr];
+        while (dr > 0 && p.s.dseg_dom[dr - 1] == d) --dr;  // at most SALT_MAX_GAMMA_BINS steps
         int dstart = p.s.dseg_ptr[dr];
-        if (dstart == start) return true;  // first user run of a domain run
+        if (dstart == start) return true;  // first user run of a domain
         int first = upper_index(p.s.useg_ptr, 0, n_useg, dstart);
         int idx = j - first - ((skip0 && dr == 0) ? 1 : 0);
         return idx % p.umax == 0;
@@ -246,8 +252,8 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         int a, len;
         group_range(g, &a, &len);
         int q = (len + TM - 1) / TM;
-        int d = p.s.useg_dom[grp_first[g]], gb = p.s.useg_gbin[grp_first[g]];
-        const float sc = d >= 0 ? p.dom_sc[d] * (gb >= 0 ? p.gamma[gb] : 1.f) : 0.f;
+        int d = p.s.useg_dom[grp_first[g]];
+        const float sc = d >= 0 ? p.dom_sc[d] : 0.f;
         for (int b = 0; b < q; ++b) {
             int s0 = a + (int)(((int64_t)b * len) / q);
             int s1 = a + (int)(((int64_t)(b + 1) * len) / q);
