@@ -199,16 +199,24 @@ def salt_centroid_fold(ctx, domain: int, layer: int, gamma: float, W, layout: in
     _check(_lib.salt_centroid_fold(ctx, domain, layer, float(gamma), _ptr(W), layout, _stream(stream)), ctx)
 
 
-def salt_align_loss(pairs, eps: float, loss, cosine=None, stream=None) -> None:
-    """pairs: sequence of dicts with At, B, At_c, B_c (CUDA bf16 tensors or
-    device addresses), r, rc, d_in, d_out, s, s_c.  loss / cosine: CUDA
-    float32 tensors of len(pairs) (cosine may be None)."""
-    n = len(pairs)
-    arr = (salt_align_pair * max(1, n))()
+def salt_align_pairs(pairs):
+    """The C array of salt_align_pair for a sequence of dicts with At, B,
+    At_c, B_c (CUDA bf16 tensors or device addresses), r, rc, d_in, d_out,
+    s, s_c; reusable across calls while the tensors live."""
+    arr = (salt_align_pair * max(1, len(pairs)))()
     for i, q in enumerate(pairs):
         arr[i] = salt_align_pair(_ptr(q["At"]), _ptr(q["B"]), _ptr(q["At_c"]), _ptr(q["B_c"]), int(q["r"]),
                                  int(q["rc"]), int(q["d_in"]), int(q["d_out"]), float(q["s"]), float(q["s_c"]))
-    _check(_lib.salt_align_loss(n, arr, float(eps), _ptr(loss), _ptr(cosine), _stream(stream)))
+    arr._n = len(pairs)
+    return arr
+
+
+def salt_align_loss(pairs, eps: float, loss, cosine=None, stream=None) -> None:
+    """pairs: a sequence of dicts (see salt_align_pairs) or its prepared
+    array.  loss / cosine: CUDA float32 tensors of len(pairs) (cosine may be
+    None)."""
+    arr = pairs if hasattr(pairs, "_n") else salt_align_pairs(pairs)
+    _check(_lib.salt_align_loss(arr._n, arr, float(eps), _ptr(loss), _ptr(cosine), _stream(stream)))
 
 
 class HostBuffer:
