@@ -191,9 +191,10 @@ salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, flo
 
 /*
  * The long-tail form of a request (Section "Multi-Tenant Serving": for rare
- * tasks the scaled centroid and the residual are concatenated offline into
- * one standard adapter, e.g. rank 17, served by plain heterogeneous
- * batching): write a blob of rank rc + rank whose factors are, per layer,
+ * tasks the scaled centroid and the residual are stacked ahead of time into
+ * one ordinary adapter - rank 17 in the paper's example - served like any
+ * other adapter of a mixed batch): write a blob of rank rc + rank whose
+ * factors are, per layer,
  *     At = [At_c ; At_u]           ([rc + rank][d_in_l])
  *     B  = [(s_c / s) B_c ; B_u]   ([rc + rank][d_out_l])
  * with blob scale s = s_u (s = 1 and B_u scaled by 0 when s_u == 0), so
@@ -212,9 +213,9 @@ salt_status salt_residual_blob_concat(const salt_config *config, int32_t rc, con
 
 /*
  * Fuse a scaled centroid into a base weight (Section "Multi-Tenant
- * Serving": high-frequency centroids are fused into the base weights at
- * node startup, after which their requests swap and apply only residuals:
- * build their segments with domain id -1).  For layer `layer` and pinned
+ * Serving": a much-used centroid, already scaled, may be merged into the
+ * base weights when a node starts, after which its requests swap and apply
+ * only residuals: build their segments with domain id -1).  For layer `layer` and pinned
  * domain `domain`:
  *     W += gamma * s_c(domain) * A_c B_c
  * in place, each element accumulated in fp32 and rounded once to bf16
@@ -292,7 +293,7 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg,
 
 /*
  * salt_build_segments with gamma bins (Section "Multi-Tenant Serving":
- * gamma is discretised into a few predefined bins and the frontend groups
+ * gamma takes one of a small fixed set of values (bins) and the frontend groups
  * requests by their (centroid, gamma) pair).  gamma_bins is int32[n_tokens]
  * in the same kind of memory as the other ids; each entry is -1 (no gamma:
  * the pinned s_c as is) or a bin in [0, n_gamma), and gamma[0..n_gamma)

@@ -30,7 +30,7 @@
  * equal domain and a user segment a maximal run of equal (domain, slot).
  *
  * gamma (same section): the centroid of a request is scaled by a
- * per-request coefficient taken from a few predefined bins, and requests are
+ * per-request coefficient taken from a small fixed set of values (bins), and requests are
  * grouped by their (centroid, gamma) pair.  Here gamma is a per-token factor
  * on the centroid term (1 when absent), and the grouping key is
  * (domain, gamma bin, slot); a token without a centroid has no bin.
@@ -39,7 +39,7 @@
  * between a task update Delta W and the centroid Wbar, evaluated from the
  * dense matrices entry by entry; and the fold of a scaled centroid into a
  * base weight (same section: high-frequency centroids are fused into the
- * base weights at node startup), W + gamma * s_c * A_c B_c entry by entry.
+ * base weights when a node starts), W + gamma * s_c * A_c B_c entry by entry.
  *
  * All functions here are pinned by tests/test_oracle_pins.py against the
  * dense closed form, the concatenation identity, special cases, invariants,

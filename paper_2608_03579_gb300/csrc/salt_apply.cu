@@ -3,8 +3,8 @@
 //
 // A row block (<= TM tokens of one domain, <= umax user runs, from the
 // segment builder) concatenates its factors into one stack of
-// S = rc + sum_u r_u rows, [A_c | a_u1 | a_u2 | ...] - the paper's
-// "centroid and residual concatenated into one standard adapter" identity,
+// S = rc + sum_u r_u rows, [A_c | a_u1 | a_u2 | ...] - the paper's long-tail
+// identity (centroid and residual stacked into one ordinary adapter),
 // applied per block - so each block is one dense contraction pair.
 //
 // One persistent kernel per apply, one CTA per SM, in two phases:

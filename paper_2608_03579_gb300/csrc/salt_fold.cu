@@ -1,6 +1,6 @@
 // Fold of a scaled centroid into a base weight (Section "Multi-Tenant
-// Serving": high-frequency centroids are fused into the base weights at
-// node startup; their requests then apply residuals only).
+// Serving": a much-used centroid, already scaled, may be merged into the
+// base weights when a node starts; its requests then apply residuals only).
 //
 //     W[Mdim][Ndim] += scale * P^T Q,   P = [rc][Mdim], Q = [rc][Ndim]
 //

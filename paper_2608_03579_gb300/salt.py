@@ -187,7 +187,7 @@ def salt_residual_blob_pack(d_in, d_out, rank: int, s_u: float, At_u, B_u, blob,
 def salt_residual_blob_concat(d_in, d_out, rc: int, At_c, B_c, s_c: float, rank: int, At_u, B_u, s_u: float,
                               blob, blob_bytes: int) -> None:
     """Blob of rank rc + rank holding the scaled centroid and the residual as
-    one standard adapter (the long-tail form)."""
+    one ordinary adapter (the long-tail form)."""
     cfg = make_config(d_in, d_out)
     _check(_lib.salt_residual_blob_concat(ctypes.byref(cfg), rc, _ptr(At_c), _ptr(B_c), float(s_c), rank,
                                           _ptr(At_u), _ptr(B_u), float(s_u), _ptr(blob), blob_bytes))

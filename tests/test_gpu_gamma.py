@@ -1,5 +1,5 @@
 """Gamma bins on the GPU (Section "Multi-Tenant Serving": requests are
-grouped by their (centroid, gamma) pair, gamma from a few predefined bins).
+grouped by their (centroid, gamma) pair, gamma from a small fixed set of bins).
 The grouping is compared bit for bit with the oracle; the apply with
 per-token gamma within the serving tolerance."""
 import numpy as np

@@ -1,6 +1,6 @@
 """Long-tail requests on the GPU (Section "Multi-Tenant Serving": the scaled
-centroid and the residual concatenated offline into one standard adapter,
-served by plain heterogeneous batching) and residual ranks above 16."""
+centroid and the residual stacked ahead of time into one ordinary adapter,
+served like any other adapter of a mixed batch) and residual ranks above 16."""
 import numpy as np
 import pytest
 import torch

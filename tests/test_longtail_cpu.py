@@ -1,6 +1,7 @@
 """The long-tail packer on the host (no GPU): salt_residual_blob_concat
-writes the scaled centroid and the residual as one standard adapter
-(Section "Multi-Tenant Serving": concatenated offline, e.g. rank 17)."""
+writes the scaled centroid and the residual as one ordinary adapter
+(Section "Multi-Tenant Serving": the long-tail form, rank 17 in the paper's
+example)."""
 import numpy as np
 import pytest
 

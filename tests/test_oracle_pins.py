@@ -3,7 +3,7 @@
 Each check ties the oracle to the paper or to mathematics it cannot share a
 mistake with: a hand-worked example, the dense closed form W_final = W_base +
 gamma*Wbar + delta_i (Section "Multi-Tenant Serving"), the concatenation of
-centroid and residual into one standard adapter (same section), the special
+centroid and residual into one ordinary adapter (same section), the special
 cases that reduce to plain multi-LoRA, linearity, permutation equivariance, a
 library sort for the grouping, and the adapter footprints the paper prints.
 """
@@ -115,7 +115,7 @@ def test_dense_closed_form_config0_shape(oracle_mod, wl):
 
 @pytest.mark.parametrize("seed", [3, 4])
 def test_concatenation_identity(oracle_mod, wl, seed):
-    """Centroid + residual equals one standard adapter of rank rc + r with
+    """Centroid + residual equals one ordinary adapter of rank rc + r with
     factors [A_c | a_u] and [s_c B_c ; s_u b_u] (the long-tail path of
     Section "Multi-Tenant Serving", e.g. r = 17)."""
     x, y_in, dom, slot, cents, res = _random_problem(wl, seed, p_none=0.0, rcs=(8, 4, 2), ranks=(1, 2, 1, 2, 1))
