@@ -95,3 +95,17 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     mod = importlib.util.module_from_spec(spec)
     with pytest.raises(ImportError):
         spec.loader.exec_module(mod)
+
+
+def test_align_loss_checks_arguments_before_any_cuda_call(salt_lib):
+    """salt_align_loss validates every pair on the host first; n = 0 is a no-op."""
+    base = dict(At=4096, B=8192, At_c=12288, B_c=16384, r=2, rc=8, d_in=64, d_out=64, s=1.0, s_c=1.0)
+    for kw, name in [(dict(r=0), "SALT_ERR_RANK"), (dict(rc=0), "SALT_ERR_RANK"), (dict(r=64, rc=65), "SALT_ERR_RANK"),
+                     (dict(d_in=60), "SALT_ERR_INVALID_ARG"), (dict(d_out=0), "SALT_ERR_INVALID_ARG"),
+                     (dict(B_c=0), "SALT_ERR_INVALID_ARG"), (dict(At=4098), "SALT_ERR_ALIGN")]:
+        q = dict(base)
+        q.update(kw)
+        with pytest.raises(salt_lib.SaltError) as e:
+            salt_lib.salt_align_loss([q], 1e-8, 256, None, 0)
+        assert e.value.name == name, (kw, e.value.name)
+    salt_lib.salt_align_loss([], 1e-8, 256, None, 0)
