@@ -18,10 +18,12 @@
 // (D[128 x S] += F_chunk F_chunk^T, fp32 in tensor memory); the unit writes
 // its S x S partial.  align_combine_kernel: COMBINE_CTAS CTAs per pair, each
 // over a slice of the S x S entries, sum the partials of each side over the
-// splits in split order (fp32) and form the three block sums of
-// G_in o G_out in fp64; the last CTA of a pair to finish (a counter) adds
-// the slices' sums in slice order and writes the loss, so the result does
-// not depend on timing.
+// splits in split order and form the slice's three block sums of
+// G_in o G_out (fp32: this part's fp64 rate is a small fraction of its fp32
+// rate, and the error added is far below the Gram entries' own fp32
+// accumulation error); the last CTA of a pair to finish (a counter) adds the
+// slices' sums in slice order in fp64 and writes the loss, so the result
+// does not depend on timing.
 #include "salt_async.cuh"
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
@@ -180,14 +182,14 @@ __global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_
     if (warp == 0) tmem_dealloc(tmem, 128);
 }
 
-__device__ double block_sum(double v, double *red)
+__device__ float block_sum(float v, float *red)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     if (lane == 0) red[warp] = v;
     __syncthreads();
-    double t = 0.0;
+    float t = 0.f;
     if (threadIdx.x == 0)
         for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
     __syncthreads();
@@ -208,7 +210,7 @@ __device__ __forceinline__ float split_sum(const float *part, int u0, int ks, in
 
 __global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __grid_constant__ AlignParams p)
 {
-    __shared__ double red[COMBINE_THREADS / 32];
+    __shared__ float red[COMBINE_THREADS / 32];
     __shared__ bool last;
     const int pi = blockIdx.x / COMBINE_CTAS, slice = blockIdx.x - pi * COMBINE_CTAS;
     const AlignPairP &pr = p.pair[pi];
@@ -216,13 +218,13 @@ __global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __
     const int u_in = p.unit_start[2 * pi], u_out = p.unit_start[2 * pi + 1];
     const int ks_in = pr.side[0].ks, ks_out = pr.side[1].ks;
     const int i0 = S * S * slice / COMBINE_CTAS, i1 = S * S * (slice + 1) / COMBINE_CTAS;
-    double num = 0.0, na = 0.0, nc = 0.0;
+    float num = 0.f, na = 0.f, nc = 0.f;
     for (int idx = i0 + threadIdx.x; idx < i1; idx += COMBINE_THREADS) {
         const int i = idx / S, j = idx - i * S;
         if (i >= r && j < r) continue;  // the lower cross block mirrors the upper one
         const float gi = split_sum(p.part, u_in, ks_in, idx);
         const float go = split_sum(p.part, u_out, ks_out, idx);
-        const double prod = (double)gi * (double)go;
+        const float prod = gi * go;
         if (i < r && j < r) na += prod;
         else if (i >= r) nc += prod;
         else num += prod;
@@ -241,16 +243,16 @@ __global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __
     __syncthreads();
     if (last && threadIdx.x == 0) {
         __threadfence();
-        num = na = nc = 0.0;
+        double dnum = 0.0, dna = 0.0, dnc = 0.0;
         for (int c = 0; c < COMBINE_CTAS; ++c) {
             const volatile double *q = p.sums + ((int64_t)pi * COMBINE_CTAS + c) * 3;
-            num += q[0];
-            na += q[1];
-            nc += q[2];
+            dnum += q[0];
+            dna += q[1];
+            dnc += q[2];
         }
-        const double tr = (double)pr.s * (double)pr.s_c * num;
-        const double n_dw = fabs((double)pr.s) * sqrt(fmax(na, 0.0));
-        const double n_wb = fabs((double)pr.s_c) * sqrt(fmax(nc, 0.0));
+        const double tr = (double)pr.s * (double)pr.s_c * dnum;
+        const double n_dw = fabs((double)pr.s) * sqrt(fmax(dna, 0.0));
+        const double n_wb = fabs((double)pr.s_c) * sqrt(fmax(dnc, 0.0));
         double cosv = tr / (n_dw * n_wb + (double)p.eps);
         if (*reinterpret_cast<volatile uint32_t *>(p.err) != 0u) cosv = __longlong_as_double(0x7ff8000000000000ll);
         p.loss[pi] = (float)(1.0 - cosv);
