@@ -66,6 +66,7 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--gamma-bins", action="store_true")
     ap.add_argument("--row", default="step", choices=["step", "fold", "align"])
+    ap.add_argument("--clocks-csv", default=None, help="also write the raw nvidia-smi samples of the timed region here")
     return ap.parse_args()
 
 
@@ -437,8 +438,7 @@ def run_salt(args, rank, world, local, pg):
             uuid = "GPU-" + uuid
     except Exception:
         uuid = None
-    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-    sampler = ClockSampler(uuid, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv"))
+    sampler = ClockSampler(uuid, f"{args.clocks_csv}.rank{rank}" if args.clocks_csv else None)
     barrier(pg, local)
     torch.cuda.synchronize(local)
     t_start = torch.cuda.Event(enable_timing=True)
@@ -687,7 +687,7 @@ def run_row(args, rank, world, local, pg):
         uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
     except Exception:
         pass
-    sampler = ClockSampler(uuid, os.path.join(ROOT, "gpurun_out", f"clocks_{args.row}_rank{rank}.csv"))
+    sampler = ClockSampler(uuid, f"{args.clocks_csv}.rank{rank}" if args.clocks_csv else None)
     barrier(pg, local)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with sampler:
