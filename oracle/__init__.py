@@ -47,7 +47,7 @@ def _configure(lib):
     vp = ctypes.c_void_p
     i32, i64 = ctypes.c_int32, ctypes.c_int64
     lib.oracle_apply.restype = ctypes.c_int
-    lib.oracle_apply.argtypes = [i64, i64, i64, vp, vp, vp, vp, vp,
+    lib.oracle_apply.argtypes = [i64, i64, i64, vp, vp, vp, i32, vp, vp, vp,
                                  i32, vp, vp, vp, vp,
                                  i32, vp, vp, vp, vp,
                                  i64, vp, vp]
@@ -92,10 +92,12 @@ def _ptr_array(arrs):
     return out, keep
 
 
-def apply(x, y_in, dom, slot, centroids, residuals, rows=None, gamma=None):
+def apply(x, y_in, dom, slot, centroids, residuals, rows=None, gamma=None, w_base=None, w_layout=0):
     """Evaluate one projection for the listed tokens in fp64.
 
     x: uint16 [T, d_in] (bf16 bits); y_in: uint16 [T, d_out] or None.
+    w_base: uint16 base weight, [d_in, d_out] (w_layout 0) or [d_out, d_in]
+    (w_layout 1), or None; when given, x W_base is added too.
     dom, slot: int32 [T], -1 drops the term.
     gamma: float64 [T] factor on each token's centroid term, or None (1).
     centroids: list over domains of (At [rc, d_in] uint16, B [rc, d_out] uint16, s_c)
@@ -142,20 +144,27 @@ def apply(x, y_in, dom, slot, centroids, residuals, rows=None, gamma=None):
 
     nd, rc, s_c, pAc, pBc, keep_c, d_out = table(centroids, d_out)
     ns, ru, s_u, pAu, pBu, keep_u, d_out = table(residuals, d_out)
-    if d_out is None:
-        raise ValueError("cannot infer d_out: pass y_in or a factor")
     if rows is None:
         rows_arr = None
         n_rows = T
     else:
         rows_arr = np.ascontiguousarray(rows, dtype=np.int64)
         n_rows = rows_arr.shape[0]
+    if w_base is not None:
+        w_base = np.ascontiguousarray(w_base, dtype=np.uint16)
+        if d_out is None:
+            d_out = w_base.shape[1] if w_layout == 0 else w_base.shape[0]
+        if w_base.shape != ((d_in, d_out) if w_layout == 0 else (d_out, d_in)):
+            raise ValueError("w_base shape does not match d_in, d_out and the layout")
+    if d_out is None:
+        raise ValueError("cannot infer d_out: pass y_in, a factor or w_base")
     out = np.zeros((n_rows, d_out), dtype=np.float64)
     if gamma is not None:
         gamma = np.ascontiguousarray(gamma, dtype=np.float64)
         if gamma.shape != (T,):
             raise ValueError("gamma must hold one factor per token")
     rc_ = lib.oracle_apply(T, d_in, d_out, _ptr(x), _ptr(y_in) if y_in is not None else None,
+                           _ptr(w_base) if w_base is not None else None, int(w_layout),
                            _ptr(dom), _ptr(slot), _ptr(gamma) if gamma is not None else None,
                            nd, _ptr(rc), _ptr(s_c), pAc, pBc,
                            ns, _ptr(ru), _ptr(s_u), pAu, pBu,

@@ -16,7 +16,9 @@
  *           + [d >= 0] * s_c(d) * sum_k (sum_i x[t,i] A_c[i,k]) B_c[k,j]
  *           + [u >= 0] * s_u(u) * sum_k (sum_i x[t,i] a_u[i,k]) b_u[k,j]
  *
- * where y_in already holds x W_base (the base GEMM is not on this path),
+ * where y_in already holds x W_base, or, when a base weight is passed, the
+ * base product x W_base is added here as well (y = y_in + x W_final, the
+ * whole of W_final = W_base + gamma Wbar + delta_i),
  * d is the token's domain (centroid) and u its residual slot, and -1 drops
  * the term (a token routed out of distribution falls back, Section
  * "Automated Centroid Routing", Stage 1).  A is stored transposed, At[k][i].
@@ -65,6 +67,8 @@ static double oracle_bf16_value(uint16_t h)
  *
  * x      [T][d_in]  bf16 bits, row-major
  * y_in   [T][d_out] bf16 bits (may be NULL: zeros)
+ * W_base base weight, bf16 bits, [d_in][d_out] (w_layout 0) or [d_out][d_in]
+ *        (w_layout 1), or NULL (no base term)
  * dom    [T] centroid index or -1;  slot [T] residual slot or -1
  * gamma  [T] per-token factor on the centroid term (NULL: 1 for every token)
  * For domain d: rc[d] ranks, s_c[d], At_c[d] -> [rc][d_in], B_c[d] -> [rc][d_out]
@@ -74,7 +78,7 @@ static double oracle_bf16_value(uint16_t h)
  * Returns 0, or -1 on an id outside its table.
  */
 int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
-                 const uint16_t *x, const uint16_t *y_in,
+                 const uint16_t *x, const uint16_t *y_in, const uint16_t *W_base, int32_t w_layout,
                  const int32_t *dom, const int32_t *slot, const double *gamma,
                  int32_t n_domains, const int32_t *rc, const double *s_c,
                  const uint16_t *const *At_c, const uint16_t *const *B_c,
@@ -103,6 +107,16 @@ int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
         }
         for (int64_t j = 0; j < d_out; ++j)
             out[j] = y_in ? oracle_bf16_value(y_in[t * d_out + j]) : 0.0;
+
+        /* base term: x W_base */
+        if (W_base) {
+            for (int64_t j = 0; j < d_out; ++j) {
+                double base = 0.0;
+                for (int64_t i = 0; i < d_in; ++i)
+                    base += oracle_bf16_value(xt[i]) * oracle_bf16_value(W_base[w_layout ? j * d_in + i : i * d_out + j]);
+                out[j] += base;
+            }
+        }
 
         /* centroid term: gamma * s_c * (x A_c) B_c */
         if (d >= 0) {

@@ -46,6 +46,10 @@ MUTANTS = {
     "fold_layout_ignored": ("int64_t idx = layout ? j * d_in + i : i * d_out + j;", "int64_t idx = i * d_out + j;"),
     "fold_A_transposed": ("double a = oracle_bf16_value(At_c[k * d_in + i]);\n            for (int64_t j = 0; j < d_out; ++j) row[j]",
                           "double a = oracle_bf16_value(At_c[i * rc + k]);\n            for (int64_t j = 0; j < d_out; ++j) row[j]"),
+    "base_term_dropped": ("                out[j] += base;", "                out[j] += 0.0 * base;"),
+    "base_layout_ignored": ("oracle_bf16_value(W_base[w_layout ? j * d_in + i : i * d_out + j])",
+                            "oracle_bf16_value(W_base[i * d_out + j])"),
+    "base_x_column": ("base += oracle_bf16_value(xt[i])", "base += oracle_bf16_value(xt[j % d_in])"),
     "fold_scale_dropped": ("W_out[idx] = oracle_bf16_value(W[idx]) + scale * row[j];",
                            "W_out[idx] = oracle_bf16_value(W[idx]) + row[j];"),
 }
@@ -74,6 +78,9 @@ def _checks(orc, wl):
         ("align_special", lambda: pins.test_align_special_cases(orc, wl)),
         ("fold_dense", lambda: [pins.test_fold_dense_brute_force(orc, wl, lay) for lay in (0, 1)]),
         ("fold_special", lambda: pins.test_fold_special_cases(orc, wl)),
+        ("w_final_dense", lambda: [pins.test_w_final_dense_closed_form(orc, wl, s, lay) for s, lay in ((30, 0), (31, 1))]),
+        ("w_final_layouts", lambda: pins.test_w_final_zero_base_and_layouts(orc, wl)),
+        ("w_final_fold", lambda: pins.test_w_final_fold_then_residual_only(orc, wl)),
     ]
     for name, fn in cases:
         try:

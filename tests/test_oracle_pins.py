@@ -435,3 +435,52 @@ def test_fold_special_cases(oracle_mod, wl):
     # fold then unfold returns W (in doubles, before any rounding)
     delta = oracle_mod.fold(Atc, Bc, 0.8, np.zeros_like(W), 0)
     assert np.abs((a - _val(W)) + 1.25 / 0.8 * delta).max() <= 1e-13 * np.abs(delta).max()
+
+
+# ---------------------------------------------------------------- the whole W_final (base GEMM + apply)
+@pytest.mark.parametrize("seed,layout", [(30, 0), (31, 1)])
+def test_w_final_dense_closed_form(oracle_mod, wl, seed, layout):
+    """y = y_in + x (W_base + gamma s_c A_c B_c + s_u a_u b_u), the final weight
+    of Section "Multi-Tenant Serving" materialised per token, for a base weight
+    stored either way."""
+    x, y_in, dom, slot, cents, res = _random_problem(wl, seed)
+    d_in, d_out = x.shape[1], y_in.shape[1]
+    W = wl.normal_bf16(seed, wl.stream_id(99, 50), d_in * d_out, 1 / np.sqrt(d_in)).reshape(d_in, d_out)
+    gamma = np.array([0.6, 0.8, 1.0])[(wl.uniform(seed, wl.stream_id(99, 51), x.shape[0]) * 3).astype(int) % 3]
+    ref = _dense_reference(x, y_in, dom, slot, cents, res, gamma) + _val(x) @ _val(W)
+    Wl = W if layout == 0 else np.ascontiguousarray(W.T)
+    got = oracle_mod.apply(x, y_in, dom, slot, cents, res, gamma=gamma, w_base=Wl, w_layout=layout)
+    assert np.abs(got - ref).max() <= 1e-12 * np.abs(ref).max()
+
+
+def test_w_final_zero_base_and_layouts(oracle_mod, wl):
+    x, y_in, dom, slot, cents, res = _random_problem(wl, 32)
+    d_in, d_out = x.shape[1], y_in.shape[1]
+    np.testing.assert_array_equal(
+        oracle_mod.apply(x, y_in, dom, slot, cents, res, w_base=np.zeros((d_in, d_out), np.uint16)),
+        oracle_mod.apply(x, y_in, dom, slot, cents, res))
+    W = wl.normal_bf16(32, wl.stream_id(99, 52), d_in * d_out).reshape(d_in, d_out)
+    np.testing.assert_array_equal(
+        oracle_mod.apply(x, y_in, dom, slot, cents, res, w_base=W, w_layout=0),
+        oracle_mod.apply(x, y_in, dom, slot, cents, res, w_base=np.ascontiguousarray(W.T), w_layout=1))
+
+
+def test_w_final_fold_then_residual_only(oracle_mod, wl):
+    """Folding a domain's scaled centroid into W_base and applying its tokens
+    with no centroid gives the same result as applying the centroid (small
+    integers: every sum is exact, so the equality is exact)."""
+    rng_vals = lambda sid, n: (np.floor(wl.uniform(33, wl.stream_id(99, sid), n) * 5) - 2).astype(np.float32)
+    T, d_in, d_out, rc = 6, 16, 24, 3
+    x = _bf(rng_vals(60, T * d_in).reshape(T, d_in))
+    W = _bf(rng_vals(61, d_in * d_out).reshape(d_in, d_out))
+    A = _bf(rng_vals(62, rc * d_in).reshape(rc, d_in))
+    B = _bf(rng_vals(63, rc * d_out).reshape(rc, d_out))
+    a = _bf(rng_vals(64, d_in).reshape(1, d_in))
+    b = _bf(rng_vals(65, d_out).reshape(1, d_out))
+    dom, slot = np.zeros(T, np.int32), np.zeros(T, np.int32)
+    cents, res = [(A, B, 0.5)], [(a, b, 2.0)]
+    with_centroid = oracle_mod.apply(x, None, dom, slot, cents, res, w_base=W)
+    folded = oracle_mod.fold(A, B, 0.5, W, 0)
+    assert np.all(np.abs(folded) < 256) and np.all(folded * 2 == np.round(folded * 2))  # exact in bf16
+    residual_only = oracle_mod.apply(x, None, np.full(T, -1, np.int32), slot, cents, res, w_base=_bf(folded))
+    np.testing.assert_array_equal(with_centroid, residual_only)
