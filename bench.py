@@ -344,55 +344,141 @@ class Step:
 
 
 # ----------------------------------------------------------------------------- oracle timing
-def oracle_sample(seconds_target: float, mode: str, n_layers: int, tokens: int | None = None):
-    """Time the fp64 oracle on a bounded sample of the same workload: the
-    7 projections of one layer for `tokens` tokens of the batch; scaled to
-    the 32-layer step.  Returns (tokens/s over the full step, sample text, seconds)."""
-    import oracle
-    from paper_2608_03579_gb300 import workloads as wl
-    w = wl.config4(seed=4, step=1, n_layers=1, rank16=(mode == "rank16"))
-    T = w.T
-    n = tokens or T
-    rows = np.arange(n)
-    tables = []
-    for l in range(7):
-        cents = [(w.centroid_At(d, l), w.centroid_B(d, l), 1.0) for d in range(w.n_domains)] if mode != "rank16" else []
-        used = set(int(s) for s in w.slot_ids[rows] if s >= 0)
-        res = [((w.residual_At(u, l), w.residual_B(u, l), 1.0) if u in used else None) for u in range(w.n_slots)]
-        tables.append((w.x(l, rows), w.y_in(l, rows), cents, res))
-    dom = w.dom_ids[rows] if mode != "rank16" else np.full(n, -1, np.int32)
-    t0 = time.perf_counter()
-    for (x, y, cents, res) in tables:
-        oracle.apply(x, y, dom, w.slot_ids[rows], cents, res)
-    dt = time.perf_counter() - t0
-    per_token_step = dt / n * n_layers
-    return 1.0 / per_token_step, f"{n} tokens x the 7 projections of 1 of {n_layers} layers, scaled x{n_layers}", dt
+def host_cores() -> int:
+    """Cores this process may run on (its affinity mask)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
+
+
+class OracleSampler:
+    """The fp64 oracle on a bounded sample of the step: some of the 512
+    tokens of one of the 32 layers, all 7 projections, with the tables of
+    that layer built once.  With n threads the tokens are split into n
+    disjoint slices, each evaluated by the same oracle call on its own host
+    thread (the C oracle runs outside the interpreter lock), so the oracle's
+    arithmetic is unchanged; only the tokens are shared out."""
+
+    def __init__(self, mode: str, n_layers: int):
+        import oracle
+        from paper_2608_03579_gb300 import workloads as wl
+        oracle.build()
+        self.oracle = oracle
+        w = wl.config4(seed=4, step=1, n_layers=1, rank16=(mode == "rank16"))
+        self.T, self.n_layers, self.mode = w.T, n_layers, mode
+        self.dom = w.dom_ids if mode != "rank16" else np.full(w.T, -1, np.int32)
+        self.slot = w.slot_ids
+        used = set(int(s) for s in w.slot_ids if s >= 0)
+        self.tables = []
+        for l in range(7):
+            cents = ([(w.centroid_At(d, l), w.centroid_B(d, l), 1.0) for d in range(w.n_domains)]
+                     if mode != "rank16" else [])
+            res = [((w.residual_At(u, l), w.residual_B(u, l), 1.0) if u in used else None)
+                   for u in range(w.n_slots)]
+            self.tables.append((w.x(l), w.y_in(l), cents, res))
+
+    def rows(self, n: int) -> np.ndarray:
+        """n tokens spread evenly over the batch (its domain and user mix)."""
+        n = max(1, min(n, self.T))
+        return np.unique(np.linspace(0, self.T - 1, n).round().astype(np.int64))
+
+    def run(self, n_tokens: int, threads: int = 1, repeat: int = 1):
+        """Seconds to evaluate n_tokens tokens of one layer `repeat` times on
+        `threads` threads; returns (seconds, token-layers evaluated)."""
+        rows = self.rows(n_tokens)
+        parts = [p for p in np.array_split(rows, max(1, min(threads, len(rows)))) if len(p)]
+
+        def work(part):
+            for _ in range(repeat):
+                for (x, y, cents, res) in self.tables:
+                    self.oracle.apply(x, y, self.dom, self.slot, cents, res, rows=part)
+
+        t0 = time.perf_counter()
+        if len(parts) == 1:
+            work(parts[0])
+        else:
+            ts = [threading.Thread(target=work, args=(p,)) for p in parts]
+            for t in ts:
+                t.start()
+            for t in ts:
+                t.join()
+        return time.perf_counter() - t0, len(rows) * repeat
+
+    def tokens_per_s(self, seconds: float, token_layers: int) -> float:
+        """Whole-step tokens/s: a token of the step passes all n_layers layers."""
+        return token_layers / self.n_layers / seconds
+
+    def sized(self, seconds_target: float, threads: int):
+        """(tokens, repeat) that take about seconds_target on `threads` threads:
+        up to the whole batch of one layer, then that layer repeated."""
+        dt, n = self.run(4 * threads, threads)
+        wall_per_token = dt / n
+        want = max(threads, int(seconds_target / max(wall_per_token, 1e-9)))
+        if want <= self.T:
+            return want, 1
+        return self.T, max(1, round(want / self.T))
+
+
+def cpu_baseline_line(mode: str, n_layers: int, seconds: float) -> dict:
+    """The oracle timed on the host cores, single-threaded and on every core
+    of the affinity mask; `value` and `cores` are the all-core run's."""
+    smp = OracleSampler(mode, n_layers)
+    cores = host_cores()
+    out = {}
+    for th in sorted({1, cores}):
+        n, rep = smp.sized(seconds / 2, th)
+        dt, tl = smp.run(n, th, rep)
+        out[th] = (smp.tokens_per_s(dt, tl), n, rep, dt)
+    v1, n1, r1, d1 = out[1]
+    vn, nn, rn, dn = out[cores]
+    return {"value": vn, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": (f"{nn} of the 512 tokens x the 7 projections of 1 of {n_layers} layers, x{rn}, on {cores} "
+                       f"threads ({dn:.1f} s); tokens/s = token-layers / {n_layers} / seconds; fp64 C oracle, "
+                       f"tokens split over threads"),
+            "single_thread": {"value": v1, "unit": "tokens/s", "cores": 1,
+                              "sample": f"{n1} tokens x 7 projections x 1 layer, x{r1} ({d1:.1f} s)"},
+            "cores_source": "os.sched_getaffinity"}
 
 
 # ----------------------------------------------------------------------------- main arms
 def run_reference(args, rank, world, pg):
-    """The oracle arm: the fp64 CPU oracle timed on the host cores."""
+    """The oracle arm: the fp64 CPU oracle timed on the host cores of rank 0.
+
+    Each step evaluates a bounded sample of the step (tokens of one of the 32
+    layers, all 7 projections) on every core; the line reports the steps it
+    ran, the seconds they took and the tokens they processed, and converts
+    them to whole-step tokens/s (a token of the step passes all 32 layers)."""
     if rank != 0:
         return
-    import oracle
-    oracle.build()
-    n_tok = 24
+    smp = OracleSampler(args.mode, args.layers)
+    cores = host_cores()
+    n_tok, rep = smp.sized(2.0, cores)  # about 2 s a step on every core
     for _ in range(args.warmup):
-        oracle_sample(0, args.mode, args.layers, tokens=4)
-    vals, tsum = [], 0.0
+        smp.run(max(cores, n_tok // 8), cores)
+    secs, toks = [], 0
     for _ in range(args.steps):
-        v, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=n_tok)
-        vals.append(v)
-        tsum += dt
-    value = statistics.mean(vals)
-    ms = 1000.0 * 512 / value
+        dt, n = smp.run(n_tok, cores, rep)
+        secs.append(dt)
+        toks += n
+    total = float(sum(secs))
+    value = toks / args.layers / total
+    d1, n1 = smp.run(max(1, n_tok // cores), 1)
+    v1 = smp.tokens_per_s(d1, n1)
+    sample = (f"each step: {n_tok} of the 512 tokens x the 7 projections of 1 of {args.layers} layers, x{rep}, "
+              f"on {cores} threads; tokens/s = token-layers evaluated / {args.layers} / seconds")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": WORKLOAD, "tokens_per_step": 512, "layers": args.layers,
-                       "projections": 7 * args.layers, "mode": args.mode},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": f"each step: {sample}"},
+                       "projections": 7 * args.layers, "mode": args.mode,
+                       "timed_per_step": {"tokens": n_tok, "layers": rep, "projections": 7 * rep},
+                       "step_equivalents_timed": toks / 512 / args.layers},
+            "timed_seconds": total, "tokens_layers_evaluated": toks,
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample,
+                             "single_thread": {"value": v1, "unit": "tokens/s", "cores": 1,
+                                               "sample": f"{n1} tokens x 7 projections x 1 layer ({d1:.1f} s)"},
+                             "cores_source": "os.sched_getaffinity"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -411,6 +497,30 @@ def traffic_from_profile():
     return d.get("dram_bytes_per_algorithmic_byte"), d
 
 
+class DeviceErrors:
+    """Reads (and clears) the library's device error word at checkpoints of a
+    run.  A bounded in-kernel wait that gave up (SALT_DEVERR_TIMEOUT) or an id
+    the kernels rejected means the launches of that stretch did less than the
+    claimed work, so any number measured over it is invalid."""
+
+    def __init__(self, salt_mod, ctx):
+        self.salt, self.ctx = salt_mod, ctx
+        self.seen = {}
+
+    def check(self, where: str, stream=None) -> int:
+        flags = int(self.salt.salt_get_device_error(self.ctx, stream))
+        if flags:
+            self.seen[where] = flags
+        return flags
+
+    @property
+    def valid(self) -> bool:
+        return not self.seen
+
+    def summary(self):
+        return {"valid": self.valid, "device_error_flags": {k: hex(v) for k, v in self.seen.items()}}
+
+
 def run_salt(args, rank, world, local, pg):
     import torch
     import __graft_entry__
@@ -418,6 +528,7 @@ def run_salt(args, rank, world, local, pg):
     torch.cuda.set_device(local)
     peaks, peak_kind = load_peaks()
     st = Step(args, local)
+    derr = DeviceErrors(st.salt, st.runner.ctx)
     ctx_info = st.salt.salt_ctx_get_info(st.runner.ctx)
     st.capture()
     per_group_bytes = st.apply_bytes()
@@ -429,6 +540,7 @@ def run_salt(args, rank, world, local, pg):
         st.step(s)
     st.join_side()
     torch.cuda.synchronize(local)
+    derr.check("warmup")
 
     # timed region: K whole steps
     uuid = None
@@ -456,7 +568,7 @@ def run_salt(args, rank, world, local, pg):
         torch.cuda.synchronize(local)
         time.sleep(0.2)
     ms_total = t_start.elapsed_time(t_end)
-    # per-launch durations of the last step (graph-captured event pairs)
+    derr.check("timed")
     barrier(pg, local)
     # per-launch durations of the apply kernel: a pass of whole steps right
     # after the timed region (swaps still overlapping), with an event pair on
@@ -468,6 +580,7 @@ def run_salt(args, rank, world, local, pg):
         st.join_side()
         torch.cuda.synchronize(local)
         launch_ms += np.array([a.elapsed_time(b) for (a, b) in evs])
+    derr.check("per_launch_timing")
     kernel_ms = list(launch_ms / n_prof)
     kinds = ["qkv", "o", "gate_up", "down"]
     per_kind = {}
@@ -488,6 +601,7 @@ def run_salt(args, rank, world, local, pg):
         b.record(st.comp)
     torch.cuda.synchronize(local)
     apply_only_ms = float(np.mean([a.elapsed_time(b) for (a, b) in reps]))
+    derr.check("apply_only_replays")
     apply_ms_timed = apply_only_ms
     ms_total = max_over_ranks(pg, ms_total, local)
     ms_per_step = ms_total / args.steps
@@ -537,6 +651,7 @@ def run_salt(args, rank, world, local, pg):
         st.join_side()
         e1.record(st.comp)
         torch.cuda.synchronize(local)
+        derr.check("e2e")
         e2e_ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / n_e2e
         h2d = st.x_elems * 2 + st.y_elems * 2 + 2 * st.T * 4 + st.wl_mod.C4_REGION * st.blob_bytes
         e2e = {"value": world * st.T / (e2e_ms / 1000.0), "unit": "tokens/s", "ms_per_step": e2e_ms,
@@ -562,15 +677,11 @@ def run_salt(args, rank, world, local, pg):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
-        oracle.build()
-        v1, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=8)
-        n_tok = int(max(8, min(512, 8 * args.cpu_seconds / max(dt, 1e-3))))
-        v, sample, dt = oracle_sample(0, args.mode, args.layers, tokens=n_tok)
-        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-               "sample": sample + f" ({dt:.1f} s, single-threaded fp64 C)"}
+        cpu = cpu_baseline_line(args.mode, args.layers, args.cpu_seconds)
 
+    derr.check("end")
     st.close()
+    valid = max_over_ranks(pg, 0.0 if derr.valid else 1.0, local) == 0.0
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -590,8 +701,13 @@ def run_salt(args, rank, world, local, pg):
                 "swap_ms_per_step_alone": swap_ms, "apply_only_ms_per_step": apply_only_ms,
                 "apply_kernel_by_group": per_kind,
                 "apply_launch_shape": {k: ctx_info[k] for k in ("apply_ctas", "k_splits_max", "apply_smem_bytes",
-                                                                  "block_tokens", "block_users")}}
+                                                                  "block_tokens", "block_users")},
+                **derr.summary(), "valid": valid}
         print(json.dumps(line), flush=True)
+    if not valid:
+        print("device error flags were raised during the run; its numbers are invalid: "
+              + json.dumps(derr.summary()), file=sys.stderr)
+        raise SystemExit(3)
 
 
 # ----------------------------------------------------------------------------- other rows of the path

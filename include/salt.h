@@ -370,7 +370,14 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
  * loads) instead of the segments object's workspace; the call itself
  * allocates nothing.  Limit: the batch may need at most 64 row blocks
  * (blocks hold <= 128 tokens of one domain); a larger batch returns
- * SALT_ERR_TOO_MANY_TOKENS before any device work.  The first call on a
+ * SALT_ERR_TOO_MANY_TOKENS before any device work.  The host judges this
+ * from the ids of the build: for host ids it counts the blocks each domain
+ * can need (ceil(tokens / 128) + ceil(user runs / block_users), see
+ * salt_ctx_get_info); device ids cannot be read on the host, so it uses the
+ * bound that holds for any ids, n_tokens / 128 + n_tokens / block_users +
+ * n_domains + 3, which refuses some batches that would fit (with rank-64
+ * centroids and rank-2 residuals, block_users = 32, from about 1,400 tokens
+ * with 8 domains).  The first call on a
  * device looks up the arrays' device addresses (cudaGetSymbolAddress);
  * make that first call before any stream capture.  Every call shares the
  * one set of arrays: calls that may overlap on the GPU (on different
@@ -379,6 +386,45 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
  */
 salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
                                    const void *x, void *y, salt_stream_t stream);
+
+/*
+ * Applies on activations that live in host memory (Section "Multi-Tenant
+ * Serving": the same W_final apply, for an engine whose activations of a
+ * step arrive from and return to the host).  A pipe owns n_stages device
+ * staging areas of stage_bytes each (0: room for the SALT_MAX_GROUP
+ * largest layers of the table at max_tokens tokens), one host-to-device and
+ * one device-to-host copy stream, and the events that order them.
+ * salt_host_pipe_create allocates all of it (synchronous); 2 <= n_stages
+ * <= 8 (0: 3).  The pipe belongs to ctx and must be destroyed before it.
+ */
+typedef struct salt_host_pipe salt_host_pipe;
+salt_status salt_host_pipe_create(salt_ctx *ctx, int32_t n_stages, int64_t stage_bytes, salt_host_pipe **out);
+
+/* Wait for everything the pipe enqueued, then free it.  NULL is a no-op. */
+void salt_host_pipe_destroy(salt_host_pipe *pipe);
+
+/*
+ * salt_lora_apply_grouped on host activations: x_host[i]
+ * ([n_tokens][d_in] bf16) and y_host[i] ([n_tokens][d_out] bf16, updated in
+ * place) are page-locked host buffers (SALT_ERR_NOT_PINNED_HOST otherwise),
+ * 16-byte aligned.  The call takes the pipe's next staging area, and
+ * enqueues: on the pipe's H2D stream, once the area's previous results
+ * have been copied out, one cudaMemcpyAsync per x and per y buffer; on
+ * `stream`, after those copies, the grouped apply on the staged copies; on
+ * the pipe's D2H stream, after the apply, one cudaMemcpyAsync per y back
+ * into y_host[i].  So with consecutive calls the copies in of call k + 1
+ * and the copies out of call k - 1 overlap the apply of call k.  The
+ * buffers' contents must stay unchanged (x, y) and unread (y) until the
+ * results are out: salt_host_pipe_wait.  The group's buffers must fit one
+ * staging area (SALT_ERR_INVALID_ARG otherwise).  Asynchronous.
+ */
+salt_status salt_lora_apply_host(salt_host_pipe *pipe, const salt_segments *seg, int32_t n,
+                                 const int32_t *layers, const void *const *x_host, void *const *y_host,
+                                 salt_stream_t stream);
+
+/* Make `stream` wait (asynchronously) until every result the pipe has
+ * enqueued so far is back in host memory. */
+salt_status salt_host_pipe_wait(salt_host_pipe *pipe, salt_stream_t stream);
 
 /*
  * The alignment regulariser of Phase 1 (Eq. 2), for n pairs of a task

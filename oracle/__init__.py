@@ -107,6 +107,8 @@ def apply(x, y_in, dom, slot, centroids, residuals, rows=None, gamma=None, w_bas
     Returns float64 [n_rows, d_out].
     """
     lib = _load()
+    if w_layout not in (0, 1):
+        raise ValueError(f"w_layout must be 0 ([d_in, d_out]) or 1 ([d_out, d_in]), not {w_layout!r}")
     x = np.ascontiguousarray(x, dtype=np.uint16)
     T, d_in = x.shape
     if y_in is not None:

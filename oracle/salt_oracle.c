@@ -75,7 +75,7 @@ static double oracle_bf16_value(uint16_t h)
  * For slot u:   r_u[u] ranks, s_u[u], At_u[u] -> [r][d_in],  B_u[u] -> [r][d_out]
  * rows   [n_rows] token indices to evaluate (NULL: all T tokens in order)
  * y_out  [n_rows][d_out] doubles
- * Returns 0, or -1 on an id outside its table.
+ * Returns 0, or -1 on an id outside its table or a w_layout other than 0 / 1.
  */
 int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
                  const uint16_t *x, const uint16_t *y_in, const uint16_t *W_base, int32_t w_layout,
@@ -88,6 +88,7 @@ int oracle_apply(int64_t T, int64_t d_in, int64_t d_out,
 {
     int64_t count = rows ? n_rows : T;
     double *v = NULL;
+    if (w_layout != 0 && w_layout != 1) return -1;
     int32_t max_rank = 1;
     for (int32_t d = 0; d < n_domains; ++d)
         if (rc[d] > max_rank) max_rank = rc[d];

@@ -62,18 +62,24 @@ constexpr int PRODUCER_WARPS = 7;              // expand roles: producers, one M
 constexpr int PRODUCER_THREADS = 32 * PRODUCER_WARPS;
 constexpr int EPI_WARPS = 4;
 static_assert(PRODUCER_WARPS + 1 + EPI_WARPS == APPLY_THREADS / 32, "expand warp roles cover the CTA");
-constexpr int TMEM_COLS = 256;                 // shrink: D^T (<= 128 tokens); expand: N_ACC x 64 columns
+constexpr int TMEM_COLS = 512;                 // expand: N_ACC x 64 accumulator columns; shrink: D^T at DT_COL
+constexpr int DT_COL = 256;                    // first column of the shrink accumulator (<= 128 tokens)
 constexpr int N_ACC = 4;                       // expand accumulators in tensor memory
 constexpr int KS_MAX = 16;
 constexpr int VT_ROW = VEXT_COLS * 2;          // bytes per V tile row
 constexpr int VT_BYTES = TM * VT_ROW;
+// a deferred unit stages the sums of its slice (<= TM / 2 token rows: the
+// block's non-empty splits are >= 2) in the V tile's region
+static_assert((TM / 2) * SALT_MAX_TOKEN_RANK * 4 <= VT_BYTES, "deferred reduction staging exceeds the V tile");
 static_assert(5 * 2 * TILE_BYTES + VT_BYTES <= RING_BYTES, "the expand ring must hold 5 full stages and the V tile");
 static_assert(VT_BYTES <= RING_BYTES, "V staging exceeds the ring");
 static_assert(S_MAX <= 128, "the factor stack is the 128-row UMMA operand");
 
 struct FusedInfo {
-    const uint16_t *src[S_MAX];  // stacked rows of the current block: A rows (shrink) or B rows (expand)
-    int32_t row[TM];             // x / y row of the i-th token of the block
+    const uint16_t *src[S_MAX];  // shrink: stacked A rows of the current unit's block
+    const uint16_t *esrc[S_MAX]; // expand: stacked B rows of the current run's block
+    int32_t row[TM];             // shrink: x row of the i-th token of the unit's block
+    int32_t erow[TM];            // expand: y row of the i-th token of the run's block
     int32_t ucol[TM];            // first stacked row of the token's user, -1: none
     int32_t urank[TM];
     float usu[TM];
@@ -82,11 +88,11 @@ struct FusedInfo {
     int16_t rt1[S_MAX];          //                    -> one past the last token
     int16_t rk[S_MAX];           //                    -> rank index within the user
     uint64_t bar[A_MAX_STAGES];  // shrink: per stage, its MMAs have completed
-    uint64_t bbar[2 * B_MAX_STAGES + 2 * N_ACC + 1];  // expand: full, empty per stage; acc full, acc empty; V full
+    // expand: full, empty per stage; acc full, acc empty; V full; run table published; item range published
+    uint64_t bbar[2 * B_MAX_STAGES + 2 * N_ACC + 3];
     int32_t range[4];            // expand: first item (block, unit), end item (block, unit)
     uint32_t tmem;
     uint32_t epoch;
-    int32_t last;
 };
 constexpr size_t FUSED_SMEM = 1024 + RING_BYTES + (sizeof(FusedInfo) + 127) / 128 * 128;
 static_assert(FUSED_SMEM <= 227 * 1024, "shared memory exceeds the per-block limit");
@@ -103,6 +109,12 @@ __device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar)
 __device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar)
 {
     asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+// Arrive with release semantics (CTA scope): shared-memory writes that
+// happen before it are visible to a thread whose wait sees the phase complete.
+__device__ __forceinline__ void mbar_arrive_release(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
 }
 // arrive on the mbarrier, adding `bytes` to the transaction count its phase waits for
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
@@ -209,6 +221,157 @@ __device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, in
 
 constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
 constexpr int N_QUADS = APPLY_THREADS / 128;  // full groups of 4 warps (one per TMEM lane quarter)
+constexpr int EPI_WARP0 = PRODUCER_WARPS + 1;  // first epilogue warp
+constexpr int EPI_THREADS = 32 * EPI_WARPS;
+constexpr int ROLE_THREADS = 32 * EPI_WARP0;   // producers + the MMA warp
+// named barriers (id 0 is __syncthreads)
+constexpr int BAR_EPI = 2;                     // the epilogue warps
+constexpr int BAR_ROLES = 3;                   // producers + the MMA warp
+constexpr int BAR_ALL = 4;                     // every thread (the inline unit finish)
+
+// The work of a shrink unit after its K loop, done by `nthr` threads
+// (warps first_warp .. first_warp + nthr/32 - 1, a whole number of groups of
+// four so that every TMEM lane quarter is read): with one split, V_ext
+// straight from the accumulator; otherwise the fp32 partial, the wait for
+// the other splits of the block, the reduction of this unit's slice of the
+// token rows over the splits (in split order) and the V rows written.  Then
+// the unit's rows are counted as written.  The shrink tables of the unit
+// (info.usc / usu / ucol / urank / rt0 / rt1 / rk) must still hold; Ps is
+// shared memory for the sums of the slice (its rows x PART_COLS floats).
+struct UnitGeom {
+    int unit, pair, s, b, pi, KS;
+    int M, rc, S, m_rows, nk, c0;
+};
+
+__device__ __forceinline__ UnitGeom unit_geom(const ApplyParams &p, int unit, int KS)
+{
+    UnitGeom g;
+    g.unit = unit;
+    g.KS = KS;
+    g.pair = unit / KS;
+    g.s = unit - g.pair * KS;
+    g.b = g.pair / p.n_proj;
+    g.pi = g.pair - g.b * p.n_proj;
+    const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * g.b);
+    const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * g.b + 4);
+    g.M = m0.y;
+    g.rc = m0.w;
+    g.S = g.rc + m1.x;
+    g.m_rows = ((g.M + 15) >> 4) << 4;
+    g.nk = (p.proj[g.pi].d_in + KC - 1) / KC;
+    g.c0 = split_lo(g.nk, g.s, KS);
+    return g;
+}
+
+__device__ void finish_split_unit(const ApplyParams &p, FusedInfo &info, const UnitGeom &g, uint32_t tmem,
+                                  uint32_t epoch, int first_warp, int nthr, int bar_id, float *Ps, bool &ok_all)
+{
+    const int tid = threadIdx.x - 32 * first_warp, lane = threadIdx.x & 31;
+    const int wrel = tid >> 5, q = (threadIdx.x >> 5) & 3, th = wrel >> 2, nth = nthr >> 7;
+    const int M = g.M, rc = g.rc, S = g.S, KS = g.KS, nk = g.nk;
+    const int n_pairs = SALT_MAX_GROUP * p.w.blk_cap;
+    const int64_t pidx = (int64_t)g.pi * p.w.blk_cap + g.b;
+    uint16_t *vt = p.w.vext + pidx * (TM * VEXT_COLS);
+    const int S_pad = (S + 15) & ~15;
+    const int nch = S_pad >> 3;
+    const int n_ne = min(KS, nk);  // splits with at least one chunk
+
+    // fp32 partial: token t's centroid columns, then its own user's columns
+    const int sr = q * 32 + lane;
+    int t0 = 0, t1 = 0, col = -1;  // tokens this stack row serves, its compact column
+    if (sr < rc) {
+        t1 = M;
+        col = sr;
+    } else if (sr < S) {
+        t0 = info.rt0[sr];
+        t1 = info.rt1[sr];
+        col = rc + info.rk[sr];
+    }
+    float *P = p.w.part + (int64_t)g.unit * (TM * PART_COLS);
+    for (int gg = th; gg < (g.m_rows >> 4); gg += nth) {
+        uint32_t v[16];
+        tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + DT_COL + gg * 16, v);
+        tmem_ld_wait();
+        if (col >= 0) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int t = gg * 16 + e;
+                if (t < M && t >= t0 && t < t1) P[t * PART_COLS + col] = __uint_as_float(v[e]);
+            }
+        }
+    }
+    tc_fence_before();
+    named_sync(bar_id, nthr);
+    // every split of the block stores its partial, then each reduces its own
+    // slice of the token rows over all splits, in split order
+    if (tid == 0) {
+        uint32_t *ctr = p.w.arrive + (epoch & 1) * n_pairs + pidx;
+        signal_add(ctr);
+        if (!wait_count(ctr, n_ne)) ok_all = false;
+    }
+    named_sync(bar_id, nthr);
+    // the non-empty splits: all of them unless d_in has fewer chunks than splits
+    uint32_t ne_mask = KS >= 32 ? ~0u : (1u << KS) - 1u;
+    if (nk < KS) {
+        ne_mask = 0;
+        for (int s2 = 0; s2 < KS; ++s2)
+            if (split_lo(nk, s2 + 1, KS) > split_lo(nk, s2, KS)) ne_mask |= 1u << s2;
+    }
+    const int si = nk >= KS ? g.s : g.c0;  // index among the non-empty splits
+    const int r0 = M * si / n_ne, r1 = M * (si + 1) / n_ne;
+    // sums of the slice's partial columns (centroid, then the token's own
+    // user's), in split order, staged in shared memory, then scaled, masked
+    // and written as bf16 V rows
+    constexpr int PC4 = PART_COLS / 4;
+    for (int idx = tid; idx < (r1 - r0) * PC4; idx += nthr) {
+        const int rr = idx / PC4, c4 = idx - rr * PC4, t = r0 + rr;
+        if (c4 * 4 >= rc + info.urank[t]) continue;
+        float4 v[KS_MAX];
+        const float *src = p.w.part + ((int64_t)g.pair * KS * TM + t) * PART_COLS + c4 * 4;
+#pragma unroll
+        for (int s2 = 0; s2 < KS_MAX; ++s2) {
+            v[s2] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if ((ne_mask >> s2) & 1)
+                v[s2] = __ldcg(reinterpret_cast<const float4 *>(src + (int64_t)s2 * (TM * PART_COLS)));
+        }
+        float4 acc = v[0];
+#pragma unroll
+        for (int s2 = 1; s2 < KS_MAX; ++s2) {
+            acc.x += v[s2].x;
+            acc.y += v[s2].y;
+            acc.z += v[s2].z;
+            acc.w += v[s2].w;
+        }
+        *reinterpret_cast<float4 *>(Ps + rr * PART_COLS + c4 * 4) = acc;
+    }
+    named_sync(bar_id, nthr);
+    for (int idx = tid; idx < (r1 - r0) * nch; idx += nthr) {
+        const int rr = idx / nch, ch = idx - rr * nch, t = r0 + rr;
+        const int uc = info.ucol[t], ur = info.urank[t];
+        const float us = info.usu[t], sc = info.usc[t];
+        const float *ps = Ps + rr * PART_COLS;
+        uint32_t w4[4];
+#pragma unroll
+        for (int hh = 0; hh < 4; ++hh) {
+            uint16_t v2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int c = ch * 8 + 2 * hh + e;
+                float val = 0.f;
+                if (c < rc) val = sc * ps[c];
+                else if (uc >= 0 && c >= uc && c < uc + ur) val = us * ps[rc + (c - uc)];
+                v2[e] = f_to_bf16(val);
+            }
+            w4[hh] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
+        }
+        *reinterpret_cast<uint4 *>(vt + t * VEXT_COLS + ch * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+    }
+    // the staging area becomes the V tile of a TMA load later
+    fence_async_smem();
+    // this unit's rows of the block's V tile are written
+    named_sync(bar_id, nthr);
+    if (tid == 0) signal_add(p.w.vdone + (epoch & 1) * n_pairs + pidx);
+}
 
 __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __grid_constant__ ApplyParams p)
 {
@@ -235,12 +398,36 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     const int n_units = n_bp * KS;
     const int ua = (int)((int64_t)n_units * blockIdx.x / gridDim.x);
     const int ub = (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
+
+    const uint32_t bb = smem_u32(&info.bbar[0]);
+    auto full_bar = [&](int st) { return bb + 8u * st; };
+    auto empty_bar = [&](int st) { return bb + 8u * (B_MAX_STAGES + st); };
+    auto accf_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + i); };
+    auto acce_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + N_ACC + i); };
+    const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 2 * N_ACC);
+    const uint32_t tbl_bar = vfull_bar + 8u;    // a run's table is written (producers -> epilogue)
+    const uint32_t range_bar = vfull_bar + 16u; // the CTA's item range is written
     if (warp == 2) {
         tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
         tmem_relinquish();
     }
     if (tid == 0) {
         for (int i = 0; i < A_MAX_STAGES; ++i) mbar_init(smem_u32(&info.bar[i]), 1);
+        // The expand's barriers are set up once; their phases run on across
+        // runs: item g (counted over all runs of this CTA) uses slot
+        // g % B_MAX_STAGES and accumulator g % N_ACC, the r-th run's V tile
+        // and table the r-th phases of "V full" and "table".
+        for (int st = 0; st < B_MAX_STAGES; ++st) {
+            mbar_init(full_bar(st), PRODUCER_THREADS);
+            mbar_init(empty_bar(st), 1 + EPI_WARPS);
+        }
+        for (int i = 0; i < N_ACC; ++i) {
+            mbar_init(accf_bar(i), 1);
+            mbar_init(acce_bar(i), EPI_WARPS);
+        }
+        mbar_init(vfull_bar, 1);
+        mbar_init(tbl_bar, 1);
+        mbar_init(range_bar, 1);
         mbar_fence_init();
     }
     tc_fence_before();
@@ -261,9 +448,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     };
 
     // This CTA's share of the expand items: the first (e = 0) or end (e = 1)
-    // item of its cost range, into info.range; one warp each.  Searched while
-    // the CTA waits for the other splits of its block (or at the end of the
-    // shrink phase): its dependent reads would otherwise delay the start.
+    // item of its cost range, into info.range; one warp each.  Searched by
+    // warps 0 and 1 while the other warps write the first shrink unit's
+    // tables, off the critical path.
     bool have_range = false;
     auto find_range = [&](int e) {
         const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
@@ -277,60 +464,69 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
 
     // ================================================================ shrink units
     uint32_t a_phase = 0;  // parity of the next completion of each stage barrier
+    // The CTA's last unit of a split shrink is finished by the epilogue warps
+    // while the producers already stream the first expand items.
+    bool deferred = false;
+    UnitGeom dgeom{};
     for (int unit = ua; unit < ub; ++unit) {
-        const int pair = unit / KS, s = unit - pair * KS;
-        const int b = pair / p.n_proj, pi = pair - b * p.n_proj;
-        const ApplyProj &pr = p.proj[pi];
-        const int4 m0 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b);
-        const int4 m1 = *reinterpret_cast<const int4 *>(p.blk + BLK_INTS * b + 4);
-        const int start = m0.x, M = m0.y, d = m0.z, rc = m0.w;
-        const int S = rc + m1.x;
+        const UnitGeom g = unit_geom(p, unit, KS);
+        const int b = g.b;
+        const ApplyProj &pr = p.proj[g.pi];
+        const int start = p.blk[BLK_INTS * b + BLK_START], d = p.blk[BLK_INTS * b + BLK_DOM];
+        const int M = g.M, rc = g.rc, S = g.S;
         const int d_in = pr.d_in;
-        const int nk = (d_in + KC - 1) / KC;
-        const int c0 = split_lo(nk, s, KS), n_my = split_lo(nk, s + 1, KS) - c0;
+        const int nk = g.nk;
+        const int c0 = g.c0, n_my = split_lo(nk, g.s + 1, KS) - c0;
         if (S > S_MAX || S == 0 || M <= 0 || n_my <= 0) {
-            if (S > S_MAX && s == 0 && tid == 0) atomicOr(p.err, SALT_DEVERR_RANK);
+            if (S > S_MAX && g.s == 0 && tid == 0) atomicOr(p.err, SALT_DEVERR_RANK);
             continue;
         }
         __syncthreads();  // the previous unit is done with info and the ring
-        if (tid < M) {
-            const int t = tid;
-            info.row[t] = p.perm[start + t];
-            const int uo = p.tok_uoff[start + t];
-            const int ur = p.tok_urank[start + t];
-            info.ucol[t] = uo >= 0 ? rc + uo : -1;
-            info.urank[t] = ur;
-            info.usu[t] = p.tok_su[start + t];
-            info.usc[t] = p.tok_sc[start + t];
-            if (uo >= 0) {
-                const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
-                const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
-                for (int k = 0; k < ur; ++k) {
-                    const int sr = rc + uo + k;
-                    if (sr < S_MAX) {
-                        if (head) {
-                            info.rt0[sr] = (int16_t)t;
-                            info.rk[sr] = (int16_t)k;
+        // the token and factor tables (threads 64..191); meanwhile warps 0 and
+        // 1 find the CTA's expand items
+        if (!have_range && warp < 2) {
+            find_range(warp);
+        } else if (tid >= 64 && tid < 64 + TM) {
+            const int t = tid - 64;
+            if (t < M) {
+                info.row[t] = p.perm[start + t];
+                const int uo = p.tok_uoff[start + t];
+                const int ur = p.tok_urank[start + t];
+                info.ucol[t] = uo >= 0 ? rc + uo : -1;
+                info.urank[t] = ur;
+                info.usu[t] = p.tok_su[start + t];
+                info.usc[t] = p.tok_sc[start + t];
+                if (uo >= 0) {
+                    const bool head = t == 0 || p.tok_uoff[start + t - 1] != uo;
+                    const bool tail = t == M - 1 || p.tok_uoff[start + t + 1] != uo;
+                    for (int k = 0; k < ur; ++k) {
+                        const int sr = rc + uo + k;
+                        if (sr < S_MAX) {
+                            if (head) {
+                                info.rt0[sr] = (int16_t)t;
+                                info.rk[sr] = (int16_t)k;
+                            }
+                            if (tail) info.rt1[sr] = (int16_t)(t + 1);
                         }
-                        if (tail) info.rt1[sr] = (int16_t)(t + 1);
                     }
                 }
             }
+            if (t < S) {
+                info.src[t] = t < rc ? pr.A + ((int64_t)d * p.rc_max + t) * d_in
+                                     : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (t - rc)], false);
+            }
         }
-        if (tid < S) {
-            info.src[tid] = tid < rc ? pr.A + ((int64_t)d * p.rc_max + tid) * d_in
-                                     : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (tid - rc)], false);
-        }
+        have_range = true;
         __syncthreads();
 
         // stage geometry: A = the factor stack (the 128-row UMMA M operand; rows
         // >= S are never read back), X = the block's tokens rounded to the
         // 16-row UMMA N step
-        const int m_rows = ((M + 15) >> 4) << 4;
+        const int m_rows = g.m_rows;
         const int stage_bytes = TILE_BYTES + m_rows * 128;
         const int nstage = min(A_MAX_STAGES, RING_BYTES / stage_bytes);
         const uint32_t idesc = idesc_bf16_f32(128, m_rows);
-        // each thread's 16-byte pieces of a chunk: piece j is (row (tid + j*256) / 8,
+        // each thread's 16-byte pieces of a chunk: piece j is (row (tid + j*384) / 8,
         // 16-byte column tid % 8), so one column offset serves all pieces
         const int cb = (tid & 7) * 8;
         const uint16_t *a_src[MAX_PIECES];
@@ -382,7 +578,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 const uint32_t sa = ring32 + st * stage_bytes, sx = sa + TILE_BYTES;
 #pragma unroll
                 for (int kk = 0; kk < KC / 16; ++kk)
-                    umma_bf16(tmem, sdesc_kmajor_sw128(sa + kk * 32), sdesc_kmajor_sw128(sx + kk * 32), idesc,
+                    umma_bf16(tmem + DT_COL, sdesc_kmajor_sw128(sa + kk * 32), sdesc_kmajor_sw128(sx + kk * 32), idesc,
                               (it > 0 || kk > 0) ? 1u : 0u);
                 umma_commit(smem_u32(&info.bar[st]));
             }
@@ -410,35 +606,32 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             }
         tc_fence_after();
 
-        // ---- D^T (TMEM lanes = stack rows, columns = tokens).  Warp w of the
-        // first N_QUADS groups of four reads lanes 32 (w % 4) .. + 31 and every
-        // N_QUADS-th 16-token group.
-        const int q = warp & 3, th = warp >> 2;
-        const int sr = q * 32 + lane;
-        int t0 = 0, t1 = 0, col = -1;  // tokens this stack row serves, its compact column
-        if (sr < rc) {
-            t1 = M;
-            col = sr;
-        } else if (sr < S) {
-            t0 = info.rt0[sr];
-            t1 = info.rt1[sr];
-            col = rc + info.rk[sr];
-        }
-        const int S_pad = (S + 15) & ~15;
-        const int n_ne = min(KS, nk);  // splits with at least one chunk
-        const int64_t pidx = (int64_t)pi * p.w.blk_cap + b;
-        uint16_t *vt = p.w.vext + pidx * (TM * VEXT_COLS);
-        const int nch = S_pad >> 3;
         if (KS == 1) {
-            // V_ext straight from the accumulator into the staging tile
-            for (int g = th; th < N_QUADS && g < (m_rows >> 4); g += N_QUADS) {
+            // ---- V_ext straight from the accumulator (TMEM lanes = stack rows,
+            // columns = tokens) into the staging tile.  Warp w of the first
+            // N_QUADS groups of four reads lanes 32 (w % 4) .. + 31 and every
+            // N_QUADS-th 16-token group.
+            const int q = warp & 3, th = warp >> 2;
+            const int sr = q * 32 + lane;
+            int t0 = 0, t1 = 0;  // tokens this stack row serves
+            if (sr < rc) {
+                t1 = M;
+            } else if (sr < S) {
+                t0 = info.rt0[sr];
+                t1 = info.rt1[sr];
+            }
+            const int S_pad = (S + 15) & ~15;
+            const int64_t pidx = (int64_t)g.pi * p.w.blk_cap + b;
+            uint16_t *vt = p.w.vext + pidx * (TM * VEXT_COLS);
+            const int nch = S_pad >> 3;
+            for (int gg = th; th < N_QUADS && gg < (m_rows >> 4); gg += N_QUADS) {
                 uint32_t v[16];
-                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
+                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + DT_COL + gg * 16, v);
                 tmem_ld_wait();
                 if (sr < S_pad) {
 #pragma unroll
                     for (int e = 0; e < 16; ++e) {
-                        const int t = g * 16 + e;
+                        const int t = gg * 16 + e;
                         if (t < M) {
                             float val = 0.f;
                             if (sr < rc) val = info.usc[t] * __uint_as_float(v[e]);
@@ -455,146 +648,65 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 *reinterpret_cast<uint4 *>(vt + r * VEXT_COLS + c * 8) =
                     *reinterpret_cast<const uint4 *>(Vs + r * VEXT_COLS + c * 8);
             }
+            __syncthreads();
+            if (tid == 0) signal_add(p.w.vdone + (info.epoch & 1) * n_pairs + pidx);
+        } else if (unit + 1 < ub || min(KS, nk) < 2) {
+            // a later unit of this CTA reuses the accumulator, or the slice
+            // (the whole block when d_in has one chunk) would not fit the V
+            // tile's region: finish now, all threads
+            __syncthreads();  // info.epoch is published
+            finish_split_unit(p, info, g, tmem, info.epoch, 0, APPLY_THREADS, BAR_ALL,
+                              reinterpret_cast<float *>(ring), ok_all);
         } else {
-            // fp32 partial: token t's centroid columns, then its own user's columns
-            float *P = p.w.part + (int64_t)unit * (TM * PART_COLS);
-            for (int g = th; th < N_QUADS && g < (m_rows >> 4); g += N_QUADS) {
-                uint32_t v[16];
-                tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + g * 16, v);
-                tmem_ld_wait();
-                if (col >= 0) {
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const int t = g * 16 + e;
-                        if (t < M && t >= t0 && t < t1) P[t * PART_COLS + col] = __uint_as_float(v[e]);
-                    }
-                }
-            }
-            tc_fence_before();
-            __syncthreads();
-            // every split of the block stores its partial, then each reduces
-            // its own slice of the token rows over all splits, in split order
-            if (tid == 0) {
-                uint32_t *ctr = p.w.arrive + (info.epoch & 1) * n_pairs + pidx;
-                signal_add(ctr);
-                if (!wait_count(ctr, n_ne)) ok_all = false;
-            } else if (!have_range && (warp == 1 || warp == 2)) {
-                find_range(warp - 1);  // meanwhile: this CTA's share of the expand items
-            }
-            have_range = true;
-            __syncthreads();
-            // the non-empty splits: all of them unless d_in has fewer chunks than splits
-            uint32_t ne_mask = KS >= 32 ? ~0u : (1u << KS) - 1u;
-            if (nk < KS) {
-                ne_mask = 0;
-                for (int s2 = 0; s2 < KS; ++s2)
-                    if (split_lo(nk, s2 + 1, KS) > split_lo(nk, s2, KS)) ne_mask |= 1u << s2;
-            }
-            const int si = nk >= KS ? s : c0;  // index among the non-empty splits
-            const int r0 = M * si / n_ne, r1 = M * (si + 1) / n_ne;
-            float *Ps = reinterpret_cast<float *>(ring);  // [r1 - r0][PART_COLS] sums
-            constexpr int PC4 = PART_COLS / 4;
-            for (int idx = tid; idx < (r1 - r0) * PC4; idx += APPLY_THREADS) {
-                const int rr = idx / PC4, c4 = idx - rr * PC4, t = r0 + rr;
-                if (c4 * 4 >= rc + info.urank[t]) continue;
-                float4 v[KS_MAX];
-                const float *src = p.w.part + ((int64_t)pair * KS * TM + t) * PART_COLS + c4 * 4;
-#pragma unroll
-                for (int s2 = 0; s2 < KS_MAX; ++s2) {
-                    v[s2] = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if ((ne_mask >> s2) & 1)
-                        v[s2] = __ldcg(reinterpret_cast<const float4 *>(src + (int64_t)s2 * (TM * PART_COLS)));
-                }
-                float4 acc = v[0];
-#pragma unroll
-                for (int s2 = 1; s2 < KS_MAX; ++s2) {
-                    acc.x += v[s2].x;
-                    acc.y += v[s2].y;
-                    acc.z += v[s2].z;
-                    acc.w += v[s2].w;
-                }
-                *reinterpret_cast<float4 *>(Ps + rr * PART_COLS + c4 * 4) = acc;
-            }
-            __syncthreads();
-            for (int idx = tid; idx < (r1 - r0) * nch; idx += APPLY_THREADS) {
-                const int rr = idx / nch, ch = idx - rr * nch, t = r0 + rr;
-                const int uc = info.ucol[t], ur = info.urank[t];
-                const float us = info.usu[t];
-                const float *ps = Ps + rr * PART_COLS;
-                uint32_t w4[4];
-#pragma unroll
-                for (int hh = 0; hh < 4; ++hh) {
-                    uint16_t v2[2];
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int c = ch * 8 + 2 * hh + e;
-                        float val = 0.f;
-                        if (c < rc) val = info.usc[t] * ps[c];
-                        else if (uc >= 0 && c >= uc && c < uc + ur) val = us * ps[rc + (c - uc)];
-                        v2[e] = f_to_bf16(val);
-                    }
-                    w4[hh] = (uint32_t)v2[0] | ((uint32_t)v2[1] << 16);
-                }
-                *reinterpret_cast<uint4 *>(vt + t * VEXT_COLS + ch * 8) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-            }
+            deferred = true;
+            dgeom = g;
         }
-        // this unit's rows of the block's V tile are written
-        __syncthreads();
-        if (tid == 0) signal_add(p.w.vdone + (info.epoch & 1) * n_pairs + pidx);
     }
     if (!waited) dep_wait();
-    if (!have_range && warp < 2) find_range(warp);
     tc_fence_before();
-    __syncthreads();  // the shrink phase is over: ring and tensor memory change hands
+    __syncthreads();  // the shrink phase is over: the ring changes hands
     tc_fence_after();
     const uint32_t epoch = info.epoch;
-    // the counters of the next launch start from zero (the previous launch,
-    // which used them, is complete)
-    {
-        const int nxt = ((epoch + 1) & 1) * n_pairs;
-        for (int i = blockIdx.x * APPLY_THREADS + tid; i < n_pairs; i += gridDim.x * APPLY_THREADS) {
-            p.w.arrive[nxt + i] = 0u;
-            p.w.vdone[nxt + i] = 0u;
-        }
-    }
 
     // ================================================================ expand items
     // Warp roles per run of items of one (block, projection):
     //   warps 0-6  producers: cp.async of each item's y rows and stacked B
     //              rows into a stage; each thread's copies complete on the
-    //              stage's "full" barrier; the V tile once per run;
-    //   warp 7     one thread issues the MMAs of an item into one of N_ACC
-    //              accumulators and commits them to "acc full" and "empty";
-    //   warps 8-11 epilogue: TMEM lanes 32 (w % 4) .. + 31 (one token row a
-    //              thread), the item's 64 columns: + staged y, one rounding,
-    //              store; then "acc empty" and "empty".
-    int b = info.range[0], u = info.range[1];
-    const int b_end = info.range[2], u_end = info.range[3];
+    //              stage's "full" barrier;
+    //   warp 7     one thread waits for the block's V tile to be written,
+    //              loads it (TMA), then issues the MMAs of an item into one
+    //              of N_ACC accumulators and commits them to "acc full" and
+    //              "empty";
+    //   warps 8-11 first the deferred split unit (partial, reduction, V
+    //              rows), then the epilogue: TMEM lanes 32 (w % 4) .. + 31
+    //              (one token row a thread), the item's 64 columns: + staged
+    //              y, one rounding, store; then "acc empty" and "empty".
+    // The producers do not wait for V: y and B do not depend on it, so the
+    // first items stream in while the splits are reduced.
     uint8_t *vs = ring + RING_BYTES - VT_BYTES;  // V_ext: two K-major tiles (K 0..63, 64..127)
     const uint32_t vs32 = smem_u32(vs);
     const uint32_t idesc_b = idesc_bf16_f32_bmn(TM, NC);
-    const uint32_t bb = smem_u32(&info.bbar[0]);
-    auto full_bar = [&](int st) { return bb + 8u * st; };
-    auto empty_bar = [&](int st) { return bb + 8u * (B_MAX_STAGES + st); };
-    auto accf_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + i); };
-    auto acce_bar = [&](int i) { return bb + 8u * (2 * B_MAX_STAGES + N_ACC + i); };
-    const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 2 * N_ACC);
-    // The barriers are set up once; their phases run on across runs: item g
-    // (counted over all runs of this CTA) uses slot g % B_MAX_STAGES and
-    // accumulator g % N_ACC, the r-th run's V tile the r-th phase of "V full".
-    if (tid == 0) {
-        for (int st = 0; st < B_MAX_STAGES; ++st) {
-            mbar_init(full_bar(st), PRODUCER_THREADS);
-            mbar_init(empty_bar(st), 1 + EPI_WARPS);
+    if (warp < EPI_WARP0) {
+        // the counters of the next launch start from zero (the previous
+        // launch, which used them, is complete)
+        const int nxt = ((epoch + 1) & 1) * n_pairs;
+        for (int i = blockIdx.x * ROLE_THREADS + tid; i < n_pairs; i += gridDim.x * ROLE_THREADS) {
+            p.w.arrive[nxt + i] = 0u;
+            p.w.vdone[nxt + i] = 0u;
         }
-        for (int i = 0; i < N_ACC; ++i) {
-            mbar_init(accf_bar(i), 1);
-            mbar_init(acce_bar(i), EPI_WARPS);
-        }
-        mbar_init(vfull_bar, 1);
-        mbar_fence_init();
+        if (!have_range && warp < 2) find_range(warp);
+        named_sync(BAR_ROLES, ROLE_THREADS);
+        if (tid == 0) mbar_arrive_release(range_bar);
+    } else {
+        // the sums are staged in the V tile's region, unused until this
+        // CTA's V rows (among others) are written
+        if (deferred)
+            finish_split_unit(p, info, dgeom, tmem, epoch, EPI_WARP0, EPI_THREADS, BAR_EPI,
+                              reinterpret_cast<float *>(vs), ok_all);
+        if (!mbar_wait(range_bar, 0)) ok_all = false;
     }
-    __syncthreads();
+    int b = info.range[0], u = info.range[1];
+    const int b_end = info.range[2], u_end = info.range[3];
     uint32_t g0 = 0, runs = 0;  // items and runs of this CTA so far
     while (b < b_end || (b == b_end && u < u_end)) {
         // a run: consecutive items of one (block, projection)
@@ -623,15 +735,19 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         const int bst = (m_rows + S_pad) * 128;
         const int nbs = min(B_MAX_STAGES, (RING_BYTES - VT_BYTES) / bst);
 
-        // The previous run is over in every role; its MMAs have completed (the
-        // epilogue saw each accumulator full), so the ring may take new rows.
-        __syncthreads();
-        if (tid < M) info.row[tid] = p.perm[start + tid];
-        if (tid < S) {
-            info.src[tid] = tid < rc ? pr.B + ((int64_t)d * p.rc_max + tid) * d_out
-                                     : residual_row(p, pr, p.blk_res[(int64_t)cb * S_MAX + (tid - rc)], true);
+        // The run's table: written by the producers and the MMA warp,
+        // published to the epilogue warps through "table" (the previous run
+        // is over in every role: the CTA barrier at the end of each run).
+        if (warp < EPI_WARP0) {
+            if (tid < M) info.erow[tid] = p.perm[start + tid];
+            if (tid >= TM && tid - TM < S) {
+                const int t = tid - TM;
+                info.esrc[t] = t < rc ? pr.B + ((int64_t)d * p.rc_max + t) * d_out
+                                      : residual_row(p, pr, p.blk_res[(int64_t)cb * S_MAX + (t - rc)], true);
+            }
+            named_sync(BAR_ROLES, ROLE_THREADS);
+            if (tid == 0) mbar_arrive_release(tbl_bar);
         }
-        __syncthreads();
 
         if (warp < PRODUCER_WARPS) {
             auto load_item = [&](int j) {
@@ -640,31 +756,16 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 for (int idx = tid; idx < M * 8; idx += PRODUCER_THREADS) {
                     const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
                     const bool ok = col < d_out;
-                    cp_async16(ys + swz128(r, c), pr.y + (int64_t)info.row[r] * d_out + (ok ? col : 0), ok);
+                    cp_async16(ys + swz128(r, c), pr.y + (int64_t)info.erow[r] * d_out + (ok ? col : 0), ok);
                 }
                 for (int idx = tid; idx < S_pad * 8; idx += PRODUCER_THREADS) {
                     const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
                     const bool ok = r < S && col < d_out;
-                    cp_async16(bs + swz128(r, c), ok ? info.src[r] + col : pr.y, ok);
+                    cp_async16(bs + swz128(r, c), ok ? info.esrc[r] + col : pr.y, ok);
                 }
                 cp_async_commit();
                 cp_async_arrive_noinc(full_bar((g0 + j) % B_MAX_STAGES));
             };
-            // V first: once every row of the block's tile is written, two TMA
-            // tile loads (K 0..63 and 64..127, each straight into the K-major
-            // 128-byte-swizzled layout) complete on "V full" by byte count.
-            // Issued before the item copies, it does not wait behind them.
-            if (tid == 0) {
-                const int n_ne = min(KS, (pr.d_in + KC - 1) / KC);
-                if (!wait_count(p.w.vdone + (epoch & 1) * n_pairs + ((int64_t)pi * p.w.blk_cap + cb), n_ne))
-                    ok_all = false;
-                fence_proxy_async_global();  // the tile was written through the generic proxy
-                const int row0 = (int)(((int64_t)pi * p.w.blk_cap + cb) * TM);
-                mbar_expect_tx(vfull_bar, 2 * TILE_BYTES);
-                tma_load_2d(vs32, &p.w.vmap, 0, row0, vfull_bar);
-                tma_load_2d(vs32 + TILE_BYTES, &p.w.vmap, 64, row0, vfull_bar);
-            }
-            named_sync(1, PRODUCER_THREADS);  // the item copies go out after V
             const int npre = min(n, nbs);
             for (int j = 0; j < npre; ++j) load_item(j);
             for (int j = npre; j < n; ++j) {
@@ -676,11 +777,22 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             cp_async_wait<0>();
         } else if (warp == PRODUCER_WARPS) {
             if (lane == 0) {
+                // V: once every row of the block's tile is written, two TMA tile
+                // loads (K 0..63 and 64..127, each straight into the K-major
+                // 128-byte-swizzled layout) complete on "V full" by byte count.
+                const int n_ne = min(KS, (pr.d_in + KC - 1) / KC);
+                const int64_t pidx = (int64_t)pi * p.w.blk_cap + cb;
+                if (!wait_count(p.w.vdone + (epoch & 1) * n_pairs + pidx, n_ne)) ok_all = false;
+                fence_proxy_async_global();  // the tile was written through the generic proxy
+                const int row0 = (int)(pidx * TM);
+                mbar_expect_tx(vfull_bar, 2 * TILE_BYTES);
+                tma_load_2d(vs32, &p.w.vmap, 0, row0, vfull_bar);
+                tma_load_2d(vs32 + TILE_BYTES, &p.w.vmap, 64, row0, vfull_bar);
                 if (!mbar_wait(vfull_bar, runs & 1)) ok_all = false;
                 for (int j = 0; j < n; ++j) {
-                    const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g % N_ACC;
-                    if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
-                    if (g >= N_ACC && !mbar_wait(acce_bar(buf), ((g / N_ACC) - 1) & 1)) ok_all = false;
+                    const uint32_t gi = g0 + j, slot = gi % B_MAX_STAGES, buf = gi % N_ACC;
+                    if (!mbar_wait(full_bar(slot), (gi / B_MAX_STAGES) & 1)) ok_all = false;
+                    if (gi >= N_ACC && !mbar_wait(acce_bar(buf), ((gi / N_ACC) - 1) & 1)) ok_all = false;
                     fence_async_smem();
                     tc_fence_after();
                     const uint32_t sb = ring32 + (j % nbs) * bst + m_rows * 128;
@@ -693,12 +805,20 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             }
             __syncwarp();
         } else {
+            if (!mbar_wait(tbl_bar, runs & 1)) ok_all = false;
             const int q = warp & 3;
             const int row = q * 32 + lane;
+            // the y rows this thread stores: 8 lanes per 128-byte row piece, 4 rows per store
+            int32_t srow[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int r = q * 32 + i * 4 + (lane >> 3);
+                srow[i] = r < M ? info.erow[r] : -1;
+            }
             for (int j = 0; j < n; ++j) {
-                const uint32_t g = g0 + j, slot = g % B_MAX_STAGES, buf = g % N_ACC;
+                const uint32_t gi = g0 + j, slot = gi % B_MAX_STAGES, buf = gi % N_ACC;
                 const int st = j % nbs;
-                if (!mbar_wait(accf_bar(buf), (g / N_ACC) & 1)) ok_all = false;
+                if (!mbar_wait(accf_bar(buf), (gi / N_ACC) & 1)) ok_all = false;
                 tc_fence_after();
                 uint32_t acc[64];
                 const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + buf * NC;
@@ -709,7 +829,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 __syncwarp();
                 if (lane == 0) mbar_arrive_relaxed(acce_bar(buf));
                 // the staged y rows of the item (its "full" phase has completed)
-                if (!mbar_wait(full_bar(slot), (g / B_MAX_STAGES) & 1)) ok_all = false;
+                if (!mbar_wait(full_bar(slot), (gi / B_MAX_STAGES) & 1)) ok_all = false;
                 // y + delta, rounded once, back into the staged tile (this
                 // thread's row) ...
                 uint8_t *ysp = ring + st * bst;
@@ -735,17 +855,16 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                             make_uint4(yv[4 * c], yv[4 * c + 1], yv[4 * c + 2], yv[4 * c + 3]);
                 }
                 __syncwarp();
-                // ... then the warp's 32 rows go out whole: 8 lanes per
-                // 128-byte row piece, 4 rows per store (all reads first)
+                // ... then the warp's 32 rows go out whole (all reads first)
                 {
                     uint4 vv[8];
                     int64_t off[8];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         const int r = q * 32 + i * 4 + (lane >> 3), c = lane & 7, col = n0 + c * 8;
-                        const bool ok = r < M && col < d_out;
+                        const bool ok = srow[i] >= 0 && col < d_out;
                         vv[i] = ok ? *reinterpret_cast<const uint4 *>(ysp + swz128(r, c)) : make_uint4(0u, 0u, 0u, 0u);
-                        off[i] = ok ? (int64_t)info.row[r] * d_out + col : -1;
+                        off[i] = ok ? (int64_t)srow[i] * d_out + col : -1;
                     }
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
@@ -757,6 +876,10 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         }
         g0 += n;
         ++runs;
+        // the run is over in every role: its MMAs have completed (the epilogue
+        // saw each accumulator full), so the ring, the V tile and the run
+        // table may take the next run's rows
+        __syncthreads();
     }
     tc_fence_before();
     __syncthreads();
@@ -779,6 +902,8 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
 // memory that exists from module load to process exit (no allocation at run
 // time).  Zero-initialised.
 __device__ __align__(256) uint16_t g_static_vext[STATIC_APPLY_BLOCKS * TM * VEXT_COLS];
+static_assert(sizeof(g_static_vext) == (size_t)1 * STATIC_APPLY_BLOCKS * TM * VEXT_COLS * 2,
+              "the static V tiles are the extent the static tensor map encodes (one projection)");
 __device__ __align__(256) float g_static_part[STATIC_PART_CAP * TM * PART_COLS];
 __device__ __align__(256) uint32_t g_static_arrive[2 * SALT_MAX_GROUP * STATIC_APPLY_BLOCKS];
 __device__ __align__(256) uint32_t g_static_vdone[2 * SALT_MAX_GROUP * STATIC_APPLY_BLOCKS];
@@ -822,6 +947,7 @@ cudaError_t apply_static_workspace(ApplyWork *out)
         if ((e = cudaGetSymbolAddress(&f, g_static_seq)) != cudaSuccess) return e;
         w.vext = static_cast<uint16_t *>(a);
         w.blk_cap = STATIC_APPLY_BLOCKS;
+        w.max_group = 1;  // one projection per call: the V array holds exactly these tiles
         w.part = static_cast<float *>(b);
         w.part_cap = STATIC_PART_CAP;
         w.arrive = static_cast<uint32_t *>(c);
@@ -851,7 +977,8 @@ cudaError_t apply_encode_vmap(ApplyWork &w)
             encode = reinterpret_cast<Encode>(fn);
         }
     }
-    const cuuint64_t dims[2] = {(cuuint64_t)VEXT_COLS, (cuuint64_t)SALT_MAX_GROUP * w.blk_cap * TM};
+    if (w.max_group < 1 || w.max_group > SALT_MAX_GROUP || w.blk_cap < 1) return cudaErrorInvalidValue;
+    const cuuint64_t dims[2] = {(cuuint64_t)VEXT_COLS, (cuuint64_t)w.max_group * w.blk_cap * TM};
     const cuuint64_t strides[1] = {(cuuint64_t)VEXT_COLS * 2};
     const cuuint32_t box[2] = {64, (cuuint32_t)TM};
     const cuuint32_t es[2] = {1, 1};

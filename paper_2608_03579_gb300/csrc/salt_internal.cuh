@@ -85,8 +85,9 @@ struct ApplyWork {
     // TMA map of vext as a 2-D bf16 tensor [rows][VEXT_COLS], box 64 x TM,
     // 128-byte swizzle (the K-major UMMA layout of a V tile half)
     alignas(64) CUtensorMap vmap;
-    uint16_t *vext;        // [SALT_MAX_GROUP * blk_cap * TM * VEXT_COLS]
+    uint16_t *vext;        // [max_group * blk_cap * TM * VEXT_COLS]
     int32_t blk_cap;
+    int32_t max_group;     // projections per launch the V tiles are sized for (vmap covers exactly these)
     float *part;           // [part_cap * TM * PART_COLS]
     int32_t part_cap;
     uint32_t *arrive;      // [2 * SALT_MAX_GROUP * blk_cap]
@@ -145,7 +146,8 @@ struct ApplyParams {
     uint32_t *err;
 };
 
-// Encode w.vmap for w.vext and w.blk_cap (host; once per workspace).
+// Encode w.vmap over the max_group * blk_cap V tiles of w.vext (host; once
+// per workspace).
 cudaError_t apply_encode_vmap(ApplyWork &w);
 
 // Kernel launchers (defined next to the kernels).

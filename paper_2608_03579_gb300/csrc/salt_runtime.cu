@@ -14,6 +14,7 @@
 #include <string>
 #include <vector>
 #include <algorithm>
+#include <functional>
 #include <map>
 #include <mutex>
 
@@ -71,6 +72,21 @@ struct salt_segments {
     std::vector<cudaStream_t> use_streams;     // build stream + apply streams since the build
     cudaEvent_t built_ev = nullptr;
     cudaEvent_t tmp_ev = nullptr;
+};
+
+// Staging and copy streams of applies on host activations.
+struct salt_host_pipe {
+    salt_ctx *ctx = nullptr;
+    int n_stages = 0;
+    int64_t stage_bytes = 0;
+    std::vector<uint8_t *> stage;              // device staging areas
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    std::vector<cudaEvent_t> in_ready;         // staged copies in (H2D stream)
+    std::vector<cudaEvent_t> applied;          // apply done (caller's stream)
+    std::vector<cudaEvent_t> out_done;         // results copied out (D2H stream)
+    std::vector<uint8_t> used;
+    int next = 0;
+    int last = -1;
 };
 
 namespace {
@@ -632,6 +648,7 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
               alloc(reinterpret_cast<int32_t **>(&seg->d.tok_sc), n) &&
               alloc(&seg->d.blk_res, (size_t)n * S_MAX);
     seg->work.blk_cap = block_bound_loose(ctx, n);
+    seg->work.max_group = SALT_MAX_GROUP;
     seg->work.part_cap = PART_CAP;
     const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
     ok = ok && cudaMalloc(&seg->work.vext, n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
@@ -981,6 +998,153 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     p.err = ctx->err_dev;
     CUDA_OR_FAIL(ctx, launch_apply(p, !seg->tables_fresh, stream));
     seg->tables_fresh = false;
+    return SALT_OK;
+}
+
+salt_status salt_host_pipe_create(salt_ctx *ctx, int32_t n_stages, int64_t stage_bytes, salt_host_pipe **out)
+{
+    if (!ctx || !out) return SALT_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (n_stages == 0) n_stages = 3;
+    if (n_stages < 2 || n_stages > 8) return fail(ctx, SALT_ERR_INVALID_ARG, "%d stages outside [2, 8]", n_stages);
+    if (stage_bytes < 0) return fail(ctx, SALT_ERR_INVALID_ARG, "negative stage size");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    if (stage_bytes == 0) {
+        // the SALT_MAX_GROUP largest layers of the table, x and y, at max_tokens
+        std::vector<int64_t> per;
+        for (int l = 0; l < ctx->n_layers; ++l) {
+            const int64_t a = ((int64_t)ctx->max_tokens * ctx->d_in[l] * 2 + 255) / 256 * 256;
+            const int64_t b = ((int64_t)ctx->max_tokens * ctx->d_out[l] * 2 + 255) / 256 * 256;
+            per.push_back(a + b);
+        }
+        std::sort(per.begin(), per.end(), std::greater<int64_t>());
+        for (size_t i = 0; i < per.size() && i < (size_t)SALT_MAX_GROUP; ++i) stage_bytes += per[i];
+    }
+    salt_host_pipe *pp = new (std::nothrow) salt_host_pipe;
+    if (!pp) return SALT_ERR_OOM;
+    pp->ctx = ctx;
+    pp->n_stages = n_stages;
+    pp->stage_bytes = (stage_bytes + 255) / 256 * 256;
+    pp->stage.assign(n_stages, nullptr);
+    pp->in_ready.assign(n_stages, nullptr);
+    pp->applied.assign(n_stages, nullptr);
+    pp->out_done.assign(n_stages, nullptr);
+    pp->used.assign(n_stages, 0);
+    bool ok = cudaStreamCreateWithFlags(&pp->h2d, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&pp->d2h, cudaStreamNonBlocking) == cudaSuccess;
+    for (int k = 0; ok && k < n_stages; ++k) {
+        ok = cudaMalloc(&pp->stage[k], (size_t)pp->stage_bytes) == cudaSuccess &&
+             cudaEventCreateWithFlags(&pp->in_ready[k], cudaEventDisableTiming) == cudaSuccess &&
+             cudaEventCreateWithFlags(&pp->applied[k], cudaEventDisableTiming) == cudaSuccess &&
+             cudaEventCreateWithFlags(&pp->out_done[k], cudaEventDisableTiming) == cudaSuccess;
+    }
+    if (!ok) {
+        cudaGetLastError();
+        salt_host_pipe_destroy(pp);
+        return fail(ctx, SALT_ERR_OOM, "host pipe allocation failed (%d stages of %lld bytes)", n_stages,
+                    (long long)pp->stage_bytes);
+    }
+    *out = pp;
+    return SALT_OK;
+}
+
+void salt_host_pipe_destroy(salt_host_pipe *pipe)
+{
+    if (!pipe) return;
+    if (pipe->ctx) set_device(pipe->ctx);
+    if (pipe->h2d) cudaStreamSynchronize(pipe->h2d);
+    if (pipe->d2h) cudaStreamSynchronize(pipe->d2h);
+    for (int k = 0; k < pipe->n_stages; ++k) {
+        if (pipe->out_done[k]) cudaEventSynchronize(pipe->out_done[k]);
+        cudaFree(pipe->stage[k]);
+        for (cudaEvent_t e : {pipe->in_ready[k], pipe->applied[k], pipe->out_done[k]})
+            if (e) cudaEventDestroy(e);
+    }
+    if (pipe->h2d) cudaStreamDestroy(pipe->h2d);
+    if (pipe->d2h) cudaStreamDestroy(pipe->d2h);
+    cudaGetLastError();
+    delete pipe;
+}
+
+salt_status salt_lora_apply_host(salt_host_pipe *pipe, const salt_segments *seg, int32_t n, const int32_t *layers,
+                                 const void *const *x_host, void *const *y_host, salt_stream_t stream_)
+{
+    if (!pipe || !pipe->ctx) return SALT_ERR_INVALID_ARG;
+    salt_ctx *ctx = pipe->ctx;
+    if (!seg || seg->ctx != ctx) return fail(ctx, SALT_ERR_INVALID_ARG, "segments of another context");
+    if (n < 1 || n > SALT_MAX_GROUP || !layers || !x_host || !y_host)
+        return fail(ctx, SALT_ERR_INVALID_ARG, "group size %d outside [1, %d] or null arrays", n, SALT_MAX_GROUP);
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (seg->stale) return fail(ctx, SALT_ERR_STALE_SEGMENTS, "a slot named by the segments was reloaded; rebuild");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    const int64_t T = seg->T;
+    int64_t off = 0;
+    int64_t xo[SALT_MAX_GROUP], yo[SALT_MAX_GROUP], xb[SALT_MAX_GROUP], yb[SALT_MAX_GROUP];
+    for (int i = 0; i < n; ++i) {
+        const int l = layers[i];
+        if (l < 0 || l >= ctx->n_layers)
+            return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", l, ctx->n_layers);
+        if (T > 0) {
+            if (!x_host[i] || !y_host[i]) return fail(ctx, SALT_ERR_INVALID_ARG, "null x or y");
+            if ((reinterpret_cast<uintptr_t>(x_host[i]) | reinterpret_cast<uintptr_t>(y_host[i])) & 15)
+                return fail(ctx, SALT_ERR_ALIGN, "x / y of group entry %d not 16-byte aligned", i);
+            for (const void *h : {static_cast<const void *>(x_host[i]), static_cast<const void *>(y_host[i])}) {
+                cudaPointerAttributes a;
+                if (cudaPointerGetAttributes(&a, h) != cudaSuccess || a.type != cudaMemoryTypeHost) {
+                    cudaGetLastError();
+                    return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "x / y of group entry %d is not page-locked host memory",
+                                i);
+                }
+            }
+        }
+        xb[i] = T * ctx->d_in[l] * 2;
+        yb[i] = T * ctx->d_out[l] * 2;
+        xo[i] = off;
+        off += (xb[i] + 255) / 256 * 256;
+        yo[i] = off;
+        off += (yb[i] + 255) / 256 * 256;
+    }
+    if (off > pipe->stage_bytes)
+        return fail(ctx, SALT_ERR_INVALID_ARG, "the group's activations (%lld bytes) exceed a staging area (%lld)",
+                    (long long)off, (long long)pipe->stage_bytes);
+    if (T == 0) return SALT_OK;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    const int k = pipe->next;
+    uint8_t *base = pipe->stage[k];
+    // copies in, once the area's previous results are out
+    if (pipe->used[k]) CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(pipe->h2d, pipe->out_done[k], 0));
+    const void *xs[SALT_MAX_GROUP];
+    void *ys[SALT_MAX_GROUP];
+    for (int i = 0; i < n; ++i) {
+        xs[i] = base + xo[i];
+        ys[i] = base + yo[i];
+        CUDA_OR_FAIL(ctx, cudaMemcpyAsync(base + xo[i], x_host[i], (size_t)xb[i], cudaMemcpyHostToDevice, pipe->h2d));
+        CUDA_OR_FAIL(ctx, cudaMemcpyAsync(base + yo[i], y_host[i], (size_t)yb[i], cudaMemcpyHostToDevice, pipe->h2d));
+    }
+    CUDA_OR_FAIL(ctx, cudaEventRecord(pipe->in_ready[k], pipe->h2d));
+    // the apply on the staged copies
+    CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(stream, pipe->in_ready[k], 0));
+    salt_status st = salt_lora_apply_grouped(ctx, seg, n, layers, xs, ys, stream_);
+    if (st != SALT_OK) return st;
+    CUDA_OR_FAIL(ctx, cudaEventRecord(pipe->applied[k], stream));
+    // copies out
+    CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(pipe->d2h, pipe->applied[k], 0));
+    for (int i = 0; i < n; ++i)
+        CUDA_OR_FAIL(ctx, cudaMemcpyAsync(y_host[i], base + yo[i], (size_t)yb[i], cudaMemcpyDeviceToHost, pipe->d2h));
+    CUDA_OR_FAIL(ctx, cudaEventRecord(pipe->out_done[k], pipe->d2h));
+    pipe->used[k] = 1;
+    pipe->last = k;
+    pipe->next = (k + 1) % pipe->n_stages;
+    return SALT_OK;
+}
+
+salt_status salt_host_pipe_wait(salt_host_pipe *pipe, salt_stream_t stream)
+{
+    if (!pipe || !pipe->ctx) return SALT_ERR_INVALID_ARG;
+    salt_ctx *ctx = pipe->ctx;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    if (pipe->last >= 0)
+        CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), pipe->out_done[pipe->last], 0));
     return SALT_OK;
 }
 

@@ -96,6 +96,10 @@ _SIGS = {
     "salt_build_segments_gamma": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp]),
     "salt_segments_export_gamma": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
     "salt_align_loss": (ctypes.c_int, [_i32, ctypes.POINTER(salt_align_pair), _f32, _vp, _vp, _vp]),
+    "salt_host_pipe_create": (ctypes.c_int, [_vp, _i32, _i64, ctypes.POINTER(_vp)]),
+    "salt_host_pipe_destroy": (None, [_vp]),
+    "salt_lora_apply_host": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
+    "salt_host_pipe_wait": (ctypes.c_int, [_vp, _vp]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -335,6 +339,41 @@ def salt_lora_apply_grouped(ctx, seg, layers, xs, ys, stream=None) -> None:
     xa = (ctypes.c_void_p * n)(*[_ptr(t) for t in xs])
     ya = (ctypes.c_void_p * n)(*[_ptr(t) for t in ys])
     _check(_lib.salt_lora_apply_grouped(ctx, seg, n, la, xa, ya, _stream(stream)), ctx)
+
+
+class HostPipe:
+    """A salt_host_pipe handle with the context it belongs to (for error messages)."""
+
+    def __init__(self, ctx, n_stages: int = 0, stage_bytes: int = 0):
+        out = _vp()
+        _check(_lib.salt_host_pipe_create(ctx, n_stages, stage_bytes, ctypes.byref(out)), ctx)
+        self.ctx, self.ptr = ctx, out.value
+
+    def close(self):
+        if self.ptr:
+            _lib.salt_host_pipe_destroy(self.ptr)
+            self.ptr = None
+
+
+def salt_host_pipe_create(ctx, n_stages: int = 0, stage_bytes: int = 0) -> HostPipe:
+    return HostPipe(ctx, n_stages, stage_bytes)
+
+
+def salt_host_pipe_destroy(pipe) -> None:
+    pipe.close()
+
+
+def salt_lora_apply_host(pipe, seg, layers, x_hosts, y_hosts, stream=None) -> None:
+    """Grouped apply on page-locked host activations (copies in, apply, copies out)."""
+    n = len(layers)
+    la = (ctypes.c_int32 * n)(*layers)
+    xa = (ctypes.c_void_p * n)(*[_ptr(t) for t in x_hosts])
+    ya = (ctypes.c_void_p * n)(*[_ptr(t) for t in y_hosts])
+    _check(_lib.salt_lora_apply_host(pipe.ptr, seg, n, la, xa, ya, _stream(stream)), pipe.ctx)
+
+
+def salt_host_pipe_wait(pipe, stream=None) -> None:
+    _check(_lib.salt_host_pipe_wait(pipe.ptr, _stream(stream)), pipe.ctx)
 
 
 def salt_selftest_wait_timeout(ctx, stream=None) -> None:

@@ -465,6 +465,27 @@ def test_w_final_zero_base_and_layouts(oracle_mod, wl):
         oracle_mod.apply(x, y_in, dom, slot, cents, res, w_base=np.ascontiguousarray(W.T), w_layout=1))
 
 
+def test_w_final_rejects_unknown_layout(oracle_mod, wl):
+    """A base-weight layout other than the two defined ones is an error in
+    both the wrapper and the C function (a typo must not fall through to the
+    transposed indexing)."""
+    import ctypes
+    x, y_in, dom, slot, cents, res = _random_problem(wl, 33)
+    d_in, d_out = x.shape[1], y_in.shape[1]
+    W = np.zeros((d_in, d_out), np.uint16)
+    for bad in (2, -1):
+        with pytest.raises(ValueError):
+            oracle_mod.apply(x, y_in, dom, slot, cents, res, w_base=W, w_layout=bad)
+    lib = oracle_mod._load()
+    z = np.zeros(1, np.int32)
+    none = np.full(1, -1, np.int32)
+    out = np.zeros(d_out, np.float64)
+    rc = lib.oracle_apply(1, d_in, d_out, x.ctypes.data, None, W.ctypes.data, 2, z.ctypes.data,
+                          none.ctypes.data, None, 0, None, None, None, None, 0, None, None, None, None,
+                          1, None, out.ctypes.data)
+    assert rc == -1
+
+
 def test_w_final_fold_then_residual_only(oracle_mod, wl):
     """Folding a domain's scaled centroid into W_base and applying its tokens
     with no centroid gives the same result as applying the centroid (small
