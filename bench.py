@@ -66,6 +66,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--gamma-bins", action="store_true")
     ap.add_argument("--row", default="step", choices=["step", "fold", "align"])
+    ap.add_argument("--config", type=int, default=4, choices=[1, 2, 3, 4],
+                    help="4: the 32-layer decode step (default); 1-3: the other serving configurations")
     ap.add_argument("--clocks-csv", default=None, help="also write the raw nvidia-smi samples of the timed region here")
     return ap.parse_args()
 
@@ -521,6 +523,85 @@ class DeviceErrors:
         return {"valid": self.valid, "device_error_flags": {k: hex(v) for k, v in self.seen.items()}}
 
 
+def host_link_rates(salt_mod, torch, device: int, nbytes: int = 1 << 30) -> dict:
+    """H2D and D2H copy rates (GB/s) of one large copy each, from and to
+    huge-page page-locked host memory, timed alone with CUDA events."""
+    hb = salt_mod.salt_host_alloc(nbytes)
+    h = hb.tensor
+    d = torch.empty(nbytes, dtype=torch.uint8, device=f"cuda:{device}")
+    s = torch.cuda.Stream(device=device)
+    out = {}
+    for name, (dst, src) in (("h2d_gbs", (d, h)), ("d2h_gbs", (h, d))):
+        with torch.cuda.stream(s):
+            dst.copy_(src, non_blocking=True)  # warm
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            for _ in range(3):
+                dst.copy_(src, non_blocking=True)
+            e1.record(s)
+        s.synchronize()
+        out[name] = 3 * nbytes / (e0.elapsed_time(e1) / 1000.0) / 1e9
+    del d
+    hb.close()
+    return out
+
+
+def step_e2e(args, st, pg, local, world, derr) -> dict:
+    """Whole steps on host activations: swaps, the segment build, then every
+    grouped apply through salt_lora_apply_host (copies in and out owned and
+    overlapped by the library); the step ends when the last y is back in
+    host memory."""
+    import torch
+    salt = st.salt
+    hb_x = salt.salt_host_alloc(st.x_elems * 2 + 4096)
+    hb_y = salt.salt_host_alloc(st.y_elems * 2 + 4096)
+    xh = hb_x.tensor[:st.x_elems * 2].view(torch.bfloat16)
+    yh = hb_y.tensor[:st.y_elems * 2].view(torch.bfloat16)
+    xh.copy_(st.x_all)
+    yh.zero_()
+    xs = [xh[st.x_off[l]:st.x_off[l] + st.T * st.w.layers[l][1]] for l in range(st.L)]
+    ys = [yh[st.y_off[l]:st.y_off[l] + st.T * st.w.layers[l][2]] for l in range(st.L)]
+    largest = max(sum(st.T * (st.w.layers[l][1] + st.w.layers[l][2]) * 2 + 512 for l in grp) for grp in st.groups)
+    pipe = salt.salt_host_pipe_create(st.runner.ctx, 3, largest)
+
+    def one(s):
+        st.swap(s)
+        st.build(s)
+        for grp in st.groups:
+            salt.salt_lora_apply_host(pipe, st.runner.seg, grp, [xs[l] for l in grp], [ys[l] for l in grp], st.comp)
+        salt.salt_host_pipe_wait(pipe, st.comp)
+
+    base = args.warmup + args.steps + 16
+    one(base)
+    st.join_side()
+    torch.cuda.synchronize(local)
+    n_e2e = max(3, min(args.steps, 10))
+    barrier(pg, local)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(st.comp)
+    for s in range(n_e2e):
+        one(base + 1 + s)
+    st.join_side()
+    e1.record(st.comp)
+    torch.cuda.synchronize(local)
+    derr.check("e2e")
+    e2e_ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / n_e2e
+    pipe.close()
+    rates = host_link_rates(salt, torch, local)
+    hb_x.close()
+    hb_y.close()
+    h2d_act = st.x_elems * 2 + st.y_elems * 2
+    h2d = h2d_act + 2 * st.T * 4 + st.wl_mod.C4_REGION * st.blob_bytes
+    d2h = st.y_elems * 2
+    return {"value": world * st.T / (e2e_ms / 1000.0), "unit": "tokens/s", "ms_per_step": e2e_ms,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "api": "salt_lora_apply_host (library-owned copies, 3 staging areas, H2D and D2H streams)",
+            "host_link": rates,
+            "bound_ms_at_host_link": {"h2d": 1000.0 * h2d / (rates["h2d_gbs"] * 1e9),
+                                      "d2h": 1000.0 * d2h / (rates["d2h_gbs"] * 1e9)}}
+
+
 def run_salt(args, rank, world, local, pg):
     import torch
     import __graft_entry__
@@ -626,39 +707,13 @@ def run_salt(args, rank, world, local, pg):
                 "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                 if peak_kind == "measured" else "fallback 6.8 TB/s"}
 
-    # e2e: host buffers, copies inside the timed region
+    # e2e: the step on host activations through the library's host pipe
+    # (salt_lora_apply_host): per grouped apply, its x and y_in are copied in,
+    # applied and y is copied out by the library, the copies of neighbouring
+    # groups overlapping the applies on two copy streams
     e2e = None
     if not args.no_e2e:
-        # host activations in huge-page page-locked memory (salt_host_alloc):
-        # ordinary pinned pages stall the copy engine under sustained transfers
-        hb = [st.salt.salt_host_alloc(n * 2) for n in (st.x_elems, st.y_elems, st.y_elems)]
-        x_host, y_host, y_out = (h.tensor.view(torch.bfloat16) for h in hb)
-        x_host.copy_(st.x_all)
-        y_host.zero_()
-        torch.cuda.synchronize(local)
-        n_e2e = max(3, min(args.steps, 10))
-        barrier(pg, local)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(st.comp)
-        for s in range(n_e2e):
-            with torch.cuda.stream(st.comp):
-                st.x_all.copy_(x_host, non_blocking=True)
-                st.y_all.copy_(y_host, non_blocking=True)
-            st.step(args.warmup + args.steps + s)
-            with torch.cuda.stream(st.comp):
-                y_out.copy_(st.y_all, non_blocking=True)
-        st.join_side()
-        e1.record(st.comp)
-        torch.cuda.synchronize(local)
-        derr.check("e2e")
-        e2e_ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / n_e2e
-        h2d = st.x_elems * 2 + st.y_elems * 2 + 2 * st.T * 4 + st.wl_mod.C4_REGION * st.blob_bytes
-        e2e = {"value": world * st.T / (e2e_ms / 1000.0), "unit": "tokens/s", "ms_per_step": e2e_ms,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(st.y_elems * 2)}
-        x_host = y_host = y_out = None
-        for h in hb:
-            h.close()
+        e2e = step_e2e(args, st, pg, local, world, derr)
 
     # swap-only and apply-only reference timings (context for the step time)
     swap_ms = None
@@ -707,6 +762,235 @@ def run_salt(args, rank, world, local, pg):
     if not valid:
         print("device error flags were raised during the run; its numbers are invalid: "
               + json.dumps(derr.summary()), file=sys.stderr)
+        raise SystemExit(3)
+
+
+# ----------------------------------------------------------------------------- the other serving configurations
+CONFIG_INFO = {
+    1: ("llama3b_decode_qkv", 28, "Llama-3.2-3B q/k/v decode, 64 tokens, 4 domains rank 16, 64 users rank 2; "
+        "one grouped q/k/v launch per layer, 28 layers (each its own factors and activations) replayed from "
+        "one CUDA graph"),
+    2: ("llama3b_prefill_mlp", 1, "Llama-3.2-3B MLP prefill, 8192 tokens in user segments of 128-1024, "
+        "4 domains rank 32, residual ranks 1 and 2; gate/up grouped, then down"),
+    3: ("llama8b_layer_decode", 8, "Llama-3.1-8B one layer (q, k, v, o, gate, up, down), 256 decode tokens, "
+        "8 domains rank 64, 256 users rank 2 drawn Zipf(1.1); 4 grouped launches per layer, 8 copies of the "
+        "layer (each its own factors and activations) replayed from one CUDA graph"),
+}
+
+
+def config_workload(wl, cfg: int):
+    """The configuration's workload with its projections repeated over R
+    layers, each with its own factors and activations (so a replay streams
+    from HBM, not L2), and the groups of every copy."""
+    w0 = wl.CONFIGS[cfg]()
+    name, R, _ = CONFIG_INFO[cfg]
+    L0 = len(w0.layers)
+    layers = [(f"c{k}.{n}", a, b) for k in range(R) for (n, a, b) in w0.layers]
+    groups = [[k * L0 + i for i in g] for k in range(R) for g in w0.group]
+    w = wl.Workload(name, w0.seed, layers, w0.n_domains, list(w0.rc), w0.n_slots, list(w0.r_u),
+                    dom_ids=w0.dom_ids, slot_ids=w0.slot_ids, group=groups)
+    return w0, w, R
+
+
+def config_cpu_baseline(w0, seconds: float) -> dict:
+    """The fp64 oracle on a bounded sample of the configuration's tokens over
+    all its projections, single-threaded and on every core (tokens split
+    over host threads); tokens/s = tokens evaluated through every projection
+    of the configuration / seconds."""
+    import oracle
+    oracle.build()
+    cores = host_cores()
+    tables = []
+    used = set(int(u) for u in w0.slot_ids if u >= 0)
+    for l in range(len(w0.layers)):
+        cents = [(w0.centroid_At(d, l), w0.centroid_B(d, l), w0.s_c[d]) for d in range(w0.n_domains)]
+        res = [((w0.residual_At(u, l), w0.residual_B(u, l), w0.s_u[u]) if u in used else None)
+               for u in range(w0.n_slots)]
+        tables.append((w0.x(l), w0.y_in(l), cents, res))
+
+    def run(rows, threads, reps=1):
+        parts = [q for q in np.array_split(rows, max(1, min(threads, len(rows)))) if len(q)]
+
+        def work(part):
+            for _ in range(reps):
+                for (x, y, cents, res) in tables:
+                    oracle.apply(x, y, w0.dom_ids, w0.slot_ids, cents, res, rows=part)
+
+        t0 = time.perf_counter()
+        ts = [threading.Thread(target=work, args=(q,)) for q in parts]
+        for t in ts:
+            t.start()
+        for t in ts:
+            t.join()
+        return time.perf_counter() - t0
+
+    out = {}
+    for th in sorted({1, cores}):
+        probe = np.linspace(0, w0.T - 1, min(w0.T, 2 * th)).round().astype(np.int64)
+        dt = run(probe, th)
+        want = (seconds / 2) / max(dt / len(probe), 1e-9)
+        n = int(max(th, min(w0.T, want)))
+        reps = max(1, int(round(want / w0.T))) if want > w0.T else 1
+        rows = np.unique(np.linspace(0, w0.T - 1, n).round().astype(np.int64))
+        dt = run(rows, th, reps)
+        out[th] = (len(rows) * reps / dt, len(rows), reps, dt)
+    (v1, n1, r1, d1), (vn, nn, rn, dn) = out[1], out[cores]
+    return {"value": vn, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{nn} of the {w0.T} tokens through all {len(w0.layers)} projections, x{rn}, on {cores} "
+                      f"threads ({dn:.1f} s); fp64 C oracle, tokens split over threads",
+            "single_thread": {"value": v1, "unit": "tokens/s", "cores": 1,
+                              "sample": f"{n1} tokens through all {len(w0.layers)} projections, x{r1} ({d1:.1f} s)"},
+            "cores_source": "os.sched_getaffinity"}
+
+
+def run_config(args, rank, world, local, pg):
+    """One JSON line for serving configuration 1, 2 or 3: the configuration's
+    grouped applies (R copies of its projections, so that every replay
+    streams from HBM) captured in one CUDA graph and replayed; the roofline
+    of the apply kernel; the oracle baseline; e2e through salt_lora_apply_host."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_03579_gb300 import salt
+    from paper_2608_03579_gb300 import workloads as wl
+    from paper_2608_03579_gb300.runner import SaltRunner
+    torch.cuda.set_device(local)
+    peaks, peak_kind = load_peaks()
+    cfg = args.config
+    w0, w, R = config_workload(wl, cfg)
+    T, L0 = w.T, len(w0.layers)
+    runner = SaltRunner(w, device=local, max_tokens=T)
+    derr = DeviceErrors(salt, runner.ctx)
+    runner.pin_centroids()
+    runner.load_slots()
+    comp = torch.cuda.Stream(device=local)
+    runner.build(stream=comp)
+    xs, ys = [], []
+    gen = torch.Generator(device=f"cuda:{local}")
+    gen.manual_seed(cfg)
+    for l in range(len(w.layers)):
+        din, dout = w.layers[l][1], w.layers[l][2]
+        xs.append(torch.randn(T, din, generator=gen, device=f"cuda:{local}").to(torch.bfloat16))
+        ys.append(torch.zeros(T, dout, dtype=torch.bfloat16, device=f"cuda:{local}"))
+
+    def applies():
+        for grp in w.group:
+            salt.salt_lora_apply_grouped(runner.ctx, runner.seg, grp, [xs[l] for l in grp], [ys[l] for l in grp], comp)
+
+    with torch.cuda.stream(comp):
+        applies()
+    torch.cuda.synchronize(local)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=comp):
+        applies()
+    for _ in range(args.warmup):
+        with torch.cuda.stream(comp):
+            graph.replay()
+    torch.cuda.synchronize(local)
+    derr.check("warmup")
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid, f"{args.clocks_csv}.rank{rank}" if args.clocks_csv else None)
+    barrier(pg, local)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with sampler:
+        time.sleep(0.2)
+        e0.record(comp)
+        for _ in range(args.steps):
+            with torch.cuda.stream(comp):
+                graph.replay()
+        e1.record(comp)
+        torch.cuda.synchronize(local)
+    derr.check("timed")
+    ms_replay = max_over_ranks(pg, e0.elapsed_time(e1), local) / args.steps
+    ms_pass = ms_replay / R  # one pass of the configuration's projections
+    value = world * T / (ms_pass / 1000.0)
+    alg = float(sum(w0.algorithmic_bytes(l) for l in range(L0)))
+    flops = float(sum(w0.algorithmic_flops(l) for l in range(L0)))
+    launches_per_pass = len(w0.group)
+    achieved = alg / (ms_pass / 1000.0) / 1e9
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+            "kernel": "salt_apply_kernel (one launch per grouped apply)",
+            "launches_per_pass": launches_per_pass, "algorithmic_bytes_per_pass": alg,
+            "avg_launch_us": 1000.0 * ms_pass / launches_per_pass,
+            "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "tensor": {"achieved_tflops": flops / (ms_pass / 1000.0) / 1e12,
+                       "peak_tflops": peaks.get("bf16_tflops"),
+                       "frac": flops / (ms_pass / 1000.0) / 1e12 / peaks["bf16_tflops"] if peaks.get("bf16_tflops") else None,
+                       "note": "algorithmic flops 2 (rc + r)(d_in + d_out) per token; the tensor cores run the "
+                               "padded stacks, more than this"}}
+    # e2e: the same pass on host activations
+    e2e = None
+    if not args.no_e2e:
+        shapes = []
+        for l in range(len(w.layers)):
+            shapes += [T * w.layers[l][1], T * w.layers[l][2]]
+        offs = np.cumsum([0] + [(n * 2 + 255) // 256 * 256 for n in shapes])
+        hb = salt.salt_host_alloc(int(offs[-1]))
+        views = [hb.tensor[int(o):int(o) + n * 2].view(torch.bfloat16) for o, n in zip(offs, shapes)]
+        xh, yh = views[0::2], views[1::2]
+        for l in range(len(w.layers)):
+            xh[l].copy_(xs[l].view(-1))
+            yh[l].zero_()
+        largest = max(sum(T * (w.layers[l][1] + w.layers[l][2]) * 2 + 512 for l in grp) for grp in w.group)
+        pipe = salt.salt_host_pipe_create(runner.ctx, 3, largest)
+
+        def host_pass():
+            for grp in w.group:
+                salt.salt_lora_apply_host(pipe, runner.seg, grp, [xh[l] for l in grp], [yh[l] for l in grp], comp)
+            salt.salt_host_pipe_wait(pipe, comp)
+
+        host_pass()
+        torch.cuda.synchronize(local)
+        n_e2e = max(2, min(args.steps, 5))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(comp)
+        for _ in range(n_e2e):
+            host_pass()
+        b.record(comp)
+        torch.cuda.synchronize(local)
+        derr.check("e2e")
+        e2e_ms_pass = max_over_ranks(pg, a.elapsed_time(b), local) / n_e2e / R
+        pipe.close()
+        hb.close()
+        rates = host_link_rates(salt, torch, local)
+        h2d = sum(T * (w0.layers[l][1] + w0.layers[l][2]) * 2 for l in range(L0))
+        d2h = sum(T * w0.layers[l][2] * 2 for l in range(L0))
+        e2e = {"value": world * T / (e2e_ms_pass / 1000.0), "unit": "tokens/s", "ms_per_pass": e2e_ms_pass,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "api": "salt_lora_apply_host", "host_link": rates,
+               "bound_ms_at_host_link": {"h2d": 1000.0 * h2d / (rates["h2d_gbs"] * 1e9),
+                                         "d2h": 1000.0 * d2h / (rates["d2h_gbs"] * 1e9)}}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = config_cpu_baseline(w0, args.cpu_seconds)
+    derr.check("end")
+    clocks = sampler.summary()
+    valid = max_over_ranks(pg, 0.0 if derr.valid else 1.0, local) == 0.0
+    runner.close()
+    if rank == 0:
+        name, _, desc = CONFIG_INFO[cfg]
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_replay, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": name, "config_index": cfg, "description": desc, "tokens": T,
+                           "projections_per_pass": L0, "copies_per_replay": R,
+                           "step": f"one CUDA-graph replay = {R} pass(es) of the configuration's projections",
+                           "algorithmic_bytes_per_pass": alg,
+                           "l2": "inputs larger than L2: each replay streams R distinct copies"
+                                 if R > 1 else "inputs larger than L2 (882 MB per pass)",
+                           "parallelism": f"replicas x{world}"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": args.steps * R * launches_per_pass,
+                "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+                **derr.summary(), "valid": valid}
+        print(json.dumps(line), flush=True)
+    if not valid:
         raise SystemExit(3)
 
 
@@ -849,6 +1133,8 @@ def main():
     try:
         if args.row != "step":
             run_row(args, rank, world, local, pg)
+        elif args.config != 4:
+            run_config(args, rank, world, local, pg)
         else:
             run_salt(args, rank, world, local, pg)
     finally:

@@ -356,6 +356,27 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
                                     void *const *y, salt_stream_t stream);
 
 /*
+ * The projection with its base weight (Section "Multi-Tenant Serving": the
+ * served weight is W_final = W_base + gamma * Wbar + delta_i): for every
+ * token t of the batch seg was built from,
+ *     y[t, :] = x[t] W_base + s_c (x[t] A_c) B_c + s_u (x[t] a_u) b_u,
+ * accumulated in fp32 and rounded once to bf16 (round to nearest even); y
+ * is written, never read (tokens with both ids -1 get x[t] W_base).  W is
+ * device bf16 in one of the layouts of salt_centroid_fold
+ * (SALT_W_IN_OUT: W[d_in][d_out]; SALT_W_OUT_IN: W[d_out][d_in]); x, W and
+ * y are 16-byte aligned, y does not overlap x or W.  Two launches on
+ * `stream`: the apply kernel writing the row blocks' V tiles into the
+ * segments workspace, then one tcgen05 kernel that runs the GEMM over
+ * 128-token tiles in grouped order and adds each overlapping row block's
+ * V * [B_c; b_u] into the same accumulator.  Asynchronous; the workspace
+ * is shared with salt_lora_apply on the same segments object (stream
+ * order keeps them apart).
+ */
+salt_status salt_lora_apply_with_base(salt_ctx *ctx, const salt_segments *seg, int32_t layer,
+                                      const void *x, const void *W, int32_t layout, void *y,
+                                      salt_stream_t stream);
+
+/*
  * salt_lora_apply for callers that cannot allocate device memory when they
  * apply - for example a serving engine whose device memory is planned up
  * front and that forbids allocations once serving starts, or code that
@@ -466,6 +487,17 @@ salt_status salt_align_loss(int32_t n, const salt_align_pair *pairs, float eps, 
  * error status instead of a hang.)
  */
 salt_status salt_selftest_wait_timeout(salt_ctx *ctx, salt_stream_t stream);
+
+/*
+ * Guard-band check (a diagnostic; the paper has no counterpart).  The
+ * library's device buffers that kernels write or gather from - the centroid
+ * arenas, the residual slot pool and, for a segments object, its V tiles and
+ * split partials - sit between two 4 KiB bands of a fixed byte pattern.
+ * This call waits for the device, reads the bands back and sets *damaged to
+ * the number of bands that changed (0 when no store or copy ran past a
+ * buffer).  seg may be NULL (context buffers only).  Synchronous.
+ */
+salt_status salt_guard_check(salt_ctx *ctx, const salt_segments *seg, int32_t *damaged);
 
 /*
  * Synchronise `stream`, then read and clear the device error word.

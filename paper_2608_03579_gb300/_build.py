@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libsalt.so")
-SOURCES = ["salt_runtime.cu", "salt_segments.cu", "salt_apply.cu", "salt_fold.cu", "salt_align.cu"]
+SOURCES = ["salt_runtime.cu", "salt_segments.cu", "salt_apply.cu", "salt_base.cu", "salt_fold.cu", "salt_align.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

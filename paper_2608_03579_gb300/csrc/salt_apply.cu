@@ -46,6 +46,7 @@
 #include <mutex>
 
 #include "salt_async.cuh"
+#include "salt_pipe.cuh"
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
 
@@ -89,54 +90,13 @@ struct FusedInfo {
     int16_t rk[S_MAX];           //                    -> rank index within the user
     uint64_t bar[A_MAX_STAGES];  // shrink: per stage, its MMAs have completed
     // expand: full, empty per stage; acc full, acc empty; V full; run table published; item range published
-    uint64_t bbar[2 * B_MAX_STAGES + 2 * N_ACC + 3];
+    uint64_t bbar[2 * B_MAX_STAGES + 2 * N_ACC + 4];
     int32_t range[4];            // expand: first item (block, unit), end item (block, unit)
     uint32_t tmem;
     uint32_t epoch;
 };
 constexpr size_t FUSED_SMEM = 1024 + RING_BYTES + (sizeof(FusedInfo) + 127) / 128 * 128;
 static_assert(FUSED_SMEM <= 227 * 1024, "shared memory exceeds the per-block limit");
-
-// arrive on the mbarrier once all of this thread's earlier cp.async copies have landed
-__device__ __forceinline__ void cp_async_arrive_noinc(uint32_t bar)
-{
-    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(bar) : "memory");
-}
-// Relaxed arrive: orders nothing by itself, so it does not wait for this
-// thread's global stores.  Used where what the barrier guards is already
-// ordered: shared-memory values consumed into registers before the arrive,
-// tensor-memory loads completed by tcgen05.wait::ld.
-__device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
-}
-// Arrive with release semantics (CTA scope): shared-memory writes that
-// happen before it are visible to a thread whose wait sees the phase complete.
-__device__ __forceinline__ void mbar_arrive_release(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
-}
-// arrive on the mbarrier, adding `bytes` to the transaction count its phase waits for
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
-}
-// 2-D TMA tile load (coordinates in elements, x first) completing on bar by bytes
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
-        "l"(map), "r"(x), "r"(y), "r"(bar)
-        : "memory");
-}
-// barrier among the first n threads of the CTA (n a multiple of 32), id 1..15
-__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory"); }
-// order global data this thread observed through the generic proxy before
-// async-proxy (TMA) reads of it
-__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;\n" ::: "memory"); }
-
-__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::); }
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p)
 {
@@ -407,6 +367,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     const uint32_t vfull_bar = bb + 8u * (2 * B_MAX_STAGES + 2 * N_ACC);
     const uint32_t tbl_bar = vfull_bar + 8u;    // a run's table is written (producers -> epilogue)
     const uint32_t range_bar = vfull_bar + 16u; // the CTA's item range is written
+    const uint32_t stg_bar = vfull_bar + 24u;   // the epilogue no longer stages in the V tile region
     if (warp == 2) {
         tmem_alloc(smem_u32(&info.tmem), TMEM_COLS);
         tmem_relinquish();
@@ -428,6 +389,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         mbar_init(vfull_bar, 1);
         mbar_init(tbl_bar, 1);
         mbar_init(range_bar, 1);
+        mbar_init(stg_bar, 1);
         mbar_fence_init();
     }
     tc_fence_before();
@@ -454,8 +416,8 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     bool have_range = false;
     auto find_range = [&](int e) {
         const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
-        int b, u;
-        item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + e) / gridDim.x, lane, b, u);
+        int b = n_blk, u = 0;  // no expand items when only the V tiles are wanted
+        if (!p.shrink_only) item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + e) / gridDim.x, lane, b, u);
         if (lane == 0) {
             info.range[2 * e] = b;
             info.range[2 * e + 1] = u;
@@ -703,6 +665,11 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         if (deferred)
             finish_split_unit(p, info, dgeom, tmem, epoch, EPI_WARP0, EPI_THREADS, BAR_EPI,
                               reinterpret_cast<float *>(vs), ok_all);
+        // the V tile region is free for the MMA warp's first V load (its
+        // staging writes go before those TMA writes)
+        fence_async_smem();
+        named_sync(BAR_EPI, EPI_THREADS);
+        if (tid == 32 * EPI_WARP0) mbar_arrive_release(stg_bar);
         if (!mbar_wait(range_bar, 0)) ok_all = false;
     }
     int b = info.range[0], u = info.range[1];
@@ -782,6 +749,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 // 128-byte-swizzled layout) complete on "V full" by byte count.
                 const int n_ne = min(KS, (pr.d_in + KC - 1) / KC);
                 const int64_t pidx = (int64_t)pi * p.w.blk_cap + cb;
+                // (the first run's load waits until the epilogue warps have
+                // staged their deferred sums in the same region)
+                if (runs == 0 && !mbar_wait(stg_bar, 0)) ok_all = false;
                 if (!wait_count(p.w.vdone + (epoch & 1) * n_pairs + pidx, n_ne)) ok_all = false;
                 fence_proxy_async_global();  // the tile was written through the generic proxy
                 const int row0 = (int)(pidx * TM);
@@ -958,6 +928,36 @@ cudaError_t apply_static_workspace(ApplyWork *out)
     }
     *out = ws[dev];
     return cudaSuccess;
+}
+
+cudaError_t encode_base_map(CUtensorMap *out, const uint16_t *W, int d_in, int d_out, int layout)
+{
+    using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+    static Encode encode = nullptr;
+    static std::mutex mu;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (!encode) {
+            void *fn = nullptr;
+            cudaDriverEntryPointQueryResult q;
+            cudaError_t e = cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &fn, cudaEnableDefault, &q);
+            if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return e != cudaSuccess ? e : cudaErrorNotSupported;
+            encode = reinterpret_cast<Encode>(fn);
+        }
+    }
+    // IN_OUT: [d_in][d_out], inner dimension N, box 64 N x 64 K;
+    // OUT_IN: [d_out][d_in], inner dimension K, box 64 K x 128 N
+    const bool in_out = layout == SALT_W_IN_OUT;
+    const cuuint64_t dims[2] = {(cuuint64_t)(in_out ? d_out : d_in), (cuuint64_t)(in_out ? d_in : d_out)};
+    const cuuint64_t strides[1] = {(cuuint64_t)(in_out ? d_out : d_in) * 2};
+    const cuuint32_t box[2] = {64, in_out ? 64u : 128u};
+    const cuuint32_t es[2] = {1, 1};
+    const CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t *>(W), dims, strides, box, es,
+                              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
 cudaError_t apply_encode_vmap(ApplyWork &w)

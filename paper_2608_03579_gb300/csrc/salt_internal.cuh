@@ -127,6 +127,7 @@ struct ApplyProj {
     int32_t d_out;
 };
 
+
 struct ApplyParams {
     ApplyProj proj[SALT_MAX_GROUP];
     int32_t n_proj;
@@ -140,11 +141,39 @@ struct ApplyParams {
     const float *tok_sc;
     const int32_t *blk_res;
     int32_t rc_max;
+    int32_t min_nk;      // fewest 64-wide d_in chunks over the group's projections (caps the K splits)
+    int32_t shrink_only; // write the V tiles of the row blocks and stop (the base-weight kernel expands)
     const uint8_t *pool;
     int64_t slot_stride;
     ApplyWork w;
     uint32_t *err;
 };
+
+// One projection of the base-weight GEMM fused with the SALT delta
+// (salt_lora_apply_with_base).
+struct BaseParams {
+    // W_base as a 2-D bf16 TMA map, 128-byte swizzle: for SALT_W_IN_OUT the
+    // tensor [d_in][d_out] with box 64 (N) x 64 (K); for SALT_W_OUT_IN the
+    // tensor [d_out][d_in] with box 64 (K) x 128 (N)
+    alignas(64) CUtensorMap wmap;
+    const uint16_t *x;       // [T][d_in]
+    uint16_t *y;             // [T][d_out], written
+    const int32_t *perm;     // grouped position -> token
+    const int32_t *blk;      // row blocks of the segments object
+    const int32_t *counts;
+    const int32_t *blk_res;
+    const uint16_t *vext;    // the blocks' V_ext tiles (projection 0 of the workspace)
+    const uint16_t *B;       // centroid arena of this layer: [n_domains][rc_max][d_out]
+    const uint8_t *pool;
+    int64_t slot_stride;
+    int64_t res_off;         // sum over earlier layers of (d_in + d_out), in elements
+    int32_t T, d_in, d_out, rc_max, w_layout, blk_cap;
+    uint32_t *err;
+};
+cudaError_t base_prepare(int device);
+cudaError_t launch_base(const BaseParams &p, cudaStream_t stream);
+// The base weight as the TMA map the fused kernel reads (host).
+cudaError_t encode_base_map(CUtensorMap *out, const uint16_t *W, int d_in, int d_out, int layout);
 
 // Encode w.vmap over the max_group * blk_cap V tiles of w.vext (host; once
 // per workspace).

@@ -35,6 +35,7 @@ struct salt_ctx {
     uint64_t layout_hash = 0;
 
     uint16_t *arenaA = nullptr, *arenaB = nullptr;
+    size_t arenaA_bytes = 0, arenaB_bytes = 0, pool_bytes = 0;
     int32_t *dom_rc_dev = nullptr;
     float *dom_sc_dev = nullptr;
     std::vector<int32_t> dom_rc;
@@ -110,6 +111,62 @@ salt_status fail(salt_ctx *ctx, salt_status s, const char *fmt, ...)
         if (e_ != cudaSuccess)                                                                     \
             return fail((ctx), SALT_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_));     \
     } while (0)
+
+// Guard bands: the device buffers the kernels write or gather from (the
+// centroid arena, the slot pool, the V tiles and the split partials) are
+// allocated with GUARD_BYTES of a fixed byte pattern before and after
+// them; salt_guard_check reads the bands back, so a store or a copy that
+// runs past one of these buffers is detected (the pool's are also the
+// bounds of every swap).
+constexpr size_t GUARD_BYTES = 4096;
+constexpr unsigned char GUARD_BYTE = 0xA5;
+
+struct Guarded {
+    void *usable;
+    size_t bytes;
+};
+
+cudaError_t guarded_malloc(void **usable, size_t bytes)
+{
+    *usable = nullptr;
+    uint8_t *base = nullptr;
+    cudaError_t e = cudaMalloc(&base, bytes + 2 * GUARD_BYTES);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaMemset(base, GUARD_BYTE, GUARD_BYTES)) != cudaSuccess ||
+        (e = cudaMemset(base + GUARD_BYTES + bytes, GUARD_BYTE, GUARD_BYTES)) != cudaSuccess) {
+        cudaFree(base);
+        return e;
+    }
+    *usable = base + GUARD_BYTES;
+    return cudaSuccess;
+}
+
+void guarded_free(void *usable)
+{
+    if (usable) cudaFree(static_cast<uint8_t *>(usable) - GUARD_BYTES);
+}
+
+// Number of the two bands of the buffer that no longer hold the pattern
+// (synchronous); -1 if they cannot be read.
+int guard_damage(const Guarded &g)
+{
+    if (!g.usable) return 0;
+    std::vector<unsigned char> h(2 * GUARD_BYTES);
+    const uint8_t *u = static_cast<const uint8_t *>(g.usable);
+    if (cudaMemcpy(h.data(), u - GUARD_BYTES, GUARD_BYTES, cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemcpy(h.data() + GUARD_BYTES, u + g.bytes, GUARD_BYTES, cudaMemcpyDeviceToHost) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    int bad = 0;
+    for (int side = 0; side < 2; ++side)
+        for (size_t i = 0; i < GUARD_BYTES; ++i)
+            if (h[side * GUARD_BYTES + i] != GUARD_BYTE) {
+                ++bad;
+                break;
+            }
+    return bad;
+}
 
 uint64_t fnv1a_layout(int n, const int32_t *din, const int32_t *dout)
 {
@@ -374,8 +431,15 @@ salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
         salt_ctx_destroy(ctx);
         return s;
     };
-    if (a > 0 && cudaMalloc(&ctx->arenaA, (size_t)a * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
-    if (b > 0 && cudaMalloc(&ctx->arenaB, (size_t)b * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    ctx->arenaA_bytes = (size_t)a * 2;
+    ctx->arenaB_bytes = (size_t)b * 2;
+    if (a > 0 && guarded_malloc(reinterpret_cast<void **>(&ctx->arenaA), ctx->arenaA_bytes) != cudaSuccess)
+        return cleanup_fail(SALT_ERR_OOM);
+    if (b > 0 && guarded_malloc(reinterpret_cast<void **>(&ctx->arenaB), ctx->arenaB_bytes) != cudaSuccess)
+        return cleanup_fail(SALT_ERR_OOM);
+    // rows of a domain beyond its pinned rank stay zero
+    if (a > 0 && cudaMemset(ctx->arenaA, 0, (size_t)a * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
+    if (b > 0 && cudaMemset(ctx->arenaB, 0, (size_t)b * 2) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
     int nd = ctx->n_domains > 0 ? ctx->n_domains : 1;
     if (cudaMalloc(&ctx->dom_rc_dev, sizeof(int32_t) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
     if (cudaMalloc(&ctx->dom_sc_dev, sizeof(float) * nd) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
@@ -385,7 +449,9 @@ salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
     ctx->dom_sc.assign(nd, 0.f);
     ctx->slot_stride = (SALT_BLOB_HEADER_BYTES + payload_elems(config, ctx->r_max) * 2 + 255) / 256 * 256;
     int ns = ctx->n_slots > 0 ? ctx->n_slots : 1;
-    if (cudaMalloc(&ctx->pool, (size_t)ctx->slot_stride * ns) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
+    ctx->pool_bytes = (size_t)ctx->slot_stride * ns;
+    if (guarded_malloc(reinterpret_cast<void **>(&ctx->pool), ctx->pool_bytes) != cudaSuccess)
+        return cleanup_fail(SALT_ERR_OOM);
     if (cudaMemset(ctx->pool, 0, (size_t)ctx->slot_stride * ns) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
     ctx->slot_rank.assign(ns, 0);
     ctx->slot_seq.assign(ns, 0);
@@ -397,7 +463,7 @@ salt_status salt_ctx_create(const salt_config *config, salt_ctx **out)
             return cleanup_fail(SALT_ERR_CUDA);
     if (cudaMalloc(&ctx->err_dev, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_OOM);
     if (cudaMemset(ctx->err_dev, 0, sizeof(uint32_t)) != cudaSuccess) return cleanup_fail(SALT_ERR_CUDA);
-    if (apply_prepare(ctx->device) != cudaSuccess) {
+    if (apply_prepare(ctx->device) != cudaSuccess || base_prepare(ctx->device) != cudaSuccess) {
         cudaGetLastError();
         return cleanup_fail(SALT_ERR_CUDA);
     }
@@ -411,11 +477,11 @@ void salt_ctx_destroy(salt_ctx *ctx)
     if (!ctx) return;
     set_device(ctx);
     cudaDeviceSynchronize();
-    cudaFree(ctx->arenaA);
-    cudaFree(ctx->arenaB);
+    guarded_free(ctx->arenaA);
+    guarded_free(ctx->arenaB);
     cudaFree(ctx->dom_rc_dev);
     cudaFree(ctx->dom_sc_dev);
-    cudaFree(ctx->pool);
+    guarded_free(ctx->pool);
     cudaFree(ctx->err_dev);
     for (cudaEvent_t e : ctx->slot_ready)
         if (e) cudaEventDestroy(e);
@@ -651,8 +717,9 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
     seg->work.max_group = SALT_MAX_GROUP;
     seg->work.part_cap = PART_CAP;
     const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
-    ok = ok && cudaMalloc(&seg->work.vext, n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
-         cudaMalloc(&seg->work.part, (size_t)PART_CAP * TM * PART_COLS * sizeof(float)) == cudaSuccess &&
+    ok = ok && guarded_malloc(reinterpret_cast<void **>(&seg->work.vext), n_pairs * TM * VEXT_COLS * 2) == cudaSuccess &&
+         guarded_malloc(reinterpret_cast<void **>(&seg->work.part), (size_t)PART_CAP * TM * PART_COLS * sizeof(float)) ==
+             cudaSuccess &&
          cudaMalloc(&seg->work.arrive, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
          cudaMalloc(&seg->work.vdone, 2 * n_pairs * sizeof(uint32_t)) == cudaSuccess &&
          cudaMalloc(&seg->work.seq, 2 * sizeof(uint32_t)) == cudaSuccess &&
@@ -694,8 +761,8 @@ void salt_segments_destroy(salt_segments *seg)
                        reinterpret_cast<int32_t *>(seg->d.tok_sc),
                        seg->d.blk_res};
     for (int32_t *p : arrs) cudaFree(p);
-    cudaFree(seg->work.vext);
-    cudaFree(seg->work.part);
+    guarded_free(seg->work.vext);
+    guarded_free(seg->work.part);
     cudaFree(seg->work.arrive);
     cudaFree(seg->work.vdone);
     cudaFree(seg->work.seq);
@@ -873,8 +940,13 @@ salt_status salt_segments_export_gamma(salt_ctx *ctx, const salt_segments *seg, 
     return SALT_OK;
 }
 
-salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, int32_t n, const int32_t *layers,
-                                    const void *const *x, void *const *y, salt_stream_t stream_)
+}  // extern "C"
+
+namespace {
+// The grouped apply; with shrink_only the launch only writes the row blocks'
+// V tiles into the segments workspace (y is not touched and may be null).
+salt_status apply_grouped(salt_ctx *ctx, const salt_segments *seg_, int32_t n, const int32_t *layers,
+                          const void *const *x, void *const *y, salt_stream_t stream_, bool shrink_only)
 {
     if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
     salt_segments *seg = const_cast<salt_segments *>(seg_);
@@ -888,7 +960,7 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
         int l = layers[i];
         if (l < 0 || l >= ctx->n_layers)
             return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", l, ctx->n_layers);
-        if (seg->T > 0 && (!x[i] || !y[i])) return fail(ctx, SALT_ERR_INVALID_ARG, "null x or y");
+        if (seg->T > 0 && (!x[i] || (!y[i] && !shrink_only))) return fail(ctx, SALT_ERR_INVALID_ARG, "null x or y");
         if ((reinterpret_cast<uintptr_t>(x[i]) | reinterpret_cast<uintptr_t>(y[i])) & 15)
             return fail(ctx, SALT_ERR_ALIGN, "x / y of group entry %d not 16-byte aligned", i);
         ApplyProj &pr = p.proj[i];
@@ -915,6 +987,8 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
         units += (p.proj[i].d_out + 63) / 64;
     }
     p.n_unit_prefix[n] = units;
+    p.min_nk = 1 << 30;
+    for (int i = 0; i < n; ++i) p.min_nk = std::min(p.min_nk, (p.proj[i].d_in + 63) / 64);
     p.perm = seg->d.perm;
     p.blk = seg->d.blk;
     p.counts = seg->d.counts;
@@ -928,10 +1002,66 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg_, in
     p.slot_stride = ctx->slot_stride;
     p.w = seg->work;
     p.err = ctx->err_dev;
+    p.shrink_only = shrink_only ? 1 : 0;
     // The first apply after a build waits for the segment kernel in full;
     // later ones overlap their table reads with the previous kernel.
     CUDA_OR_FAIL(ctx, launch_apply(p, !seg->tables_fresh, stream));
     seg->tables_fresh = false;
+    return SALT_OK;
+}
+}  // namespace
+
+extern "C" {
+
+salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int32_t n, const int32_t *layers,
+                                    const void *const *x, void *const *y, salt_stream_t stream)
+{
+    return apply_grouped(ctx, seg, n, layers, x, y, stream, false);
+}
+
+salt_status salt_lora_apply_with_base(salt_ctx *ctx, const salt_segments *seg_, int32_t layer, const void *x,
+                                      const void *W, int32_t layout, void *y, salt_stream_t stream_)
+{
+    if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
+    salt_segments *seg = const_cast<salt_segments *>(seg_);
+    if (layer < 0 || layer >= ctx->n_layers)
+        return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", layer, ctx->n_layers);
+    if (layout != SALT_W_IN_OUT && layout != SALT_W_OUT_IN) return fail(ctx, SALT_ERR_INVALID_ARG, "unknown layout %d", layout);
+    if (!seg->built) return fail(ctx, SALT_ERR_NOT_BUILT, "segments object was never built");
+    if (seg->stale) return fail(ctx, SALT_ERR_STALE_SEGMENTS, "a slot named by the segments was reloaded; rebuild");
+    if (seg->T > 0 && (!x || !W || !y)) return fail(ctx, SALT_ERR_INVALID_ARG, "null x, W or y");
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y) | reinterpret_cast<uintptr_t>(W)) & 15)
+        return fail(ctx, SALT_ERR_ALIGN, "x, W or y not 16-byte aligned");
+    if (seg->T == 0) return SALT_OK;
+    // 1. the row blocks' V tiles (shrink only)
+    const void *xs[1] = {x};
+    void *ys[1] = {nullptr};
+    salt_status st = apply_grouped(ctx, seg, 1, &layer, xs, ys, stream_, true);
+    if (st != SALT_OK) return st;
+    // 2. the base GEMM with the delta of every overlapping row block
+    BaseParams bp;
+    std::memset(&bp, 0, sizeof bp);
+    const int din = ctx->d_in[layer], dout = ctx->d_out[layer];
+    CUDA_OR_FAIL(ctx, encode_base_map(&bp.wmap, static_cast<const uint16_t *>(W), din, dout, layout));
+    bp.x = static_cast<const uint16_t *>(x);
+    bp.y = static_cast<uint16_t *>(y);
+    bp.perm = seg->d.perm;
+    bp.blk = seg->d.blk;
+    bp.counts = seg->d.counts;
+    bp.blk_res = seg->d.blk_res;
+    bp.vext = seg->work.vext;
+    bp.B = ctx->arenaB ? ctx->arenaB + ctx->b_off[layer] : nullptr;
+    bp.pool = ctx->pool;
+    bp.slot_stride = ctx->slot_stride;
+    bp.res_off = ctx->res_off[layer];
+    bp.T = seg->T;
+    bp.d_in = din;
+    bp.d_out = dout;
+    bp.rc_max = ctx->rc_max;
+    bp.w_layout = layout;
+    bp.blk_cap = seg->work.blk_cap;
+    bp.err = ctx->err_dev;
+    CUDA_OR_FAIL(ctx, launch_base(bp, static_cast<cudaStream_t>(stream_)));
     return SALT_OK;
 }
 
@@ -983,6 +1113,7 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     p.n_proj = 1;
     p.n_unit_prefix[0] = 0;
     p.n_unit_prefix[1] = (pr.d_out + 63) / 64;
+    p.min_nk = (pr.d_in + 63) / 64;
     p.perm = seg->d.perm;
     p.blk = seg->d.blk;
     p.counts = seg->d.counts;
@@ -1145,6 +1276,29 @@ salt_status salt_host_pipe_wait(salt_host_pipe *pipe, salt_stream_t stream)
     if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
     if (pipe->last >= 0)
         CUDA_OR_FAIL(ctx, cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), pipe->out_done[pipe->last], 0));
+    return SALT_OK;
+}
+
+salt_status salt_guard_check(salt_ctx *ctx, const salt_segments *seg, int32_t *damaged)
+{
+    if (!ctx || !damaged) return SALT_ERR_INVALID_ARG;
+    if (seg && seg->ctx != ctx) return fail(ctx, SALT_ERR_INVALID_ARG, "segments of another context");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    CUDA_OR_FAIL(ctx, cudaDeviceSynchronize());
+    std::vector<Guarded> bufs = {{ctx->arenaA, ctx->arenaA_bytes}, {ctx->arenaB, ctx->arenaB_bytes},
+                                 {ctx->pool, ctx->pool_bytes}};
+    if (seg) {
+        const size_t n_pairs = (size_t)SALT_MAX_GROUP * seg->work.blk_cap;
+        bufs.push_back({seg->work.vext, n_pairs * TM * VEXT_COLS * 2});
+        bufs.push_back({seg->work.part, (size_t)PART_CAP * TM * PART_COLS * sizeof(float)});
+    }
+    int bad = 0;
+    for (const Guarded &g : bufs) {
+        const int d = guard_damage(g);
+        if (d < 0) return fail(ctx, SALT_ERR_CUDA, "guard bands could not be read");
+        bad += d;
+    }
+    *damaged = bad;
     return SALT_OK;
 }
 

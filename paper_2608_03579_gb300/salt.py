@@ -100,6 +100,8 @@ _SIGS = {
     "salt_host_pipe_destroy": (None, [_vp]),
     "salt_lora_apply_host": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _vp, _vp]),
     "salt_host_pipe_wait": (ctypes.c_int, [_vp, _vp]),
+    "salt_guard_check": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
+    "salt_lora_apply_with_base": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -328,6 +330,11 @@ def salt_lora_apply(ctx, seg, layer: int, x, y, stream=None) -> None:
     _check(_lib.salt_lora_apply(ctx, seg, layer, _ptr(x), _ptr(y), _stream(stream)), ctx)
 
 
+def salt_lora_apply_with_base(ctx, seg, layer: int, x, W, layout: int, y, stream=None) -> None:
+    """y = x W_base + the SALT delta (y written, not read)."""
+    _check(_lib.salt_lora_apply_with_base(ctx, seg, layer, _ptr(x), _ptr(W), layout, _ptr(y), _stream(stream)), ctx)
+
+
 def salt_lora_apply_static(ctx, seg, layer: int, x, y, stream=None) -> None:
     """salt_lora_apply without any device allocation behind it (static scratch)."""
     _check(_lib.salt_lora_apply_static(ctx, seg, layer, _ptr(x), _ptr(y), _stream(stream)), ctx)
@@ -374,6 +381,13 @@ def salt_lora_apply_host(pipe, seg, layers, x_hosts, y_hosts, stream=None) -> No
 
 def salt_host_pipe_wait(pipe, stream=None) -> None:
     _check(_lib.salt_host_pipe_wait(pipe.ptr, _stream(stream)), pipe.ctx)
+
+
+def salt_guard_check(ctx, seg=None) -> int:
+    """Number of damaged guard bands around the library's device buffers (synchronous)."""
+    n = ctypes.c_int32(0)
+    _check(_lib.salt_guard_check(ctx, seg, ctypes.byref(n)), ctx)
+    return int(n.value)
 
 
 def salt_selftest_wait_timeout(ctx, stream=None) -> None:

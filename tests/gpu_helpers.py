@@ -45,3 +45,27 @@ def assert_close(y_bits, y_ref, what=""):
     assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} elements out of tolerance; "
                            f"worst err {err.max():.4g} (ref max {np.abs(ref).max():.4g}) at {np.unravel_index(err.argmax(), err.shape)}")
     return float((err / (np.abs(ref).max() + 1e-30)).max())
+
+
+GUARD_ELEMS = 2048          # 4 KiB of bf16 on each side of a guarded buffer
+GUARD_BITS = 0x5AA5
+
+
+def guarded_like(t):
+    """A copy of the device tensor t inside a larger buffer whose 4 KiB on
+    each side hold a fixed pattern; returns (view of the copy, buffer)."""
+    import torch
+    n = t.numel()
+    buf = torch.empty(n + 2 * GUARD_ELEMS, dtype=t.dtype, device=t.device)
+    buf.view(torch.int16).fill_(GUARD_BITS - (1 << 16) if GUARD_BITS >= (1 << 15) else GUARD_BITS)
+    view = buf[GUARD_ELEMS:GUARD_ELEMS + n].view(t.shape)
+    view.copy_(t)
+    return view, buf
+
+
+def guards_intact(buf) -> bool:
+    """True when both bands of a guarded_like buffer still hold the pattern."""
+    import torch
+    b = buf.view(torch.int16)
+    pat = GUARD_BITS - (1 << 16) if GUARD_BITS >= (1 << 15) else GUARD_BITS
+    return bool((b[:GUARD_ELEMS] == pat).all().item() and (b[-GUARD_ELEMS:] == pat).all().item())

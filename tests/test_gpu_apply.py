@@ -3,13 +3,16 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_helpers import assert_close, oracle_tables
+from gpu_helpers import assert_close, guarded_like, guards_intact, oracle_tables
 
 pytestmark = pytest.mark.gpu
 
 
 def run_gpu(wl, groups, y_mode=None, scales_c=None, repeat=1):
-    """Pin, swap every slot, build, apply each group; return {layer: y bits}."""
+    """Pin, swap every slot, build, apply each group; return {layer: y bits}.
+    Every y sits between guard bands, and the library's own guard bands
+    (centroid arenas, slot pool, V tiles, split partials) are checked after
+    the applies: a store past any of these buffers fails the test."""
     from paper_2608_03579_gb300.runner import SaltRunner, bf16_bits
     if y_mode:
         wl.y_mode = y_mode
@@ -20,12 +23,18 @@ def run_gpu(wl, groups, y_mode=None, scales_c=None, repeat=1):
         r.build()
         for grp in groups:
             xs, ys = r.alloc_xy(grp)
+            gys = [guarded_like(y) for y in ys]
+            ys = [g[0] for g in gys]
             for _ in range(repeat):
                 r.apply(grp, xs, ys)
-            for l, y in zip(grp, ys):
+            torch.cuda.synchronize()
+            for l, y, (_, buf) in zip(grp, ys, gys):
                 out[l] = bf16_bits(y)
+                assert guards_intact(buf), f"a store ran past y of layer {l}"
         torch.cuda.synchronize()
         assert r.device_error() == 0
+        from paper_2608_03579_gb300 import salt
+        assert salt.salt_guard_check(r.ctx, r.seg) == 0, "a guard band of the library's buffers changed"
     return out
 
 
