@@ -65,7 +65,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--gamma-bins", action="store_true")
-    ap.add_argument("--row", default="step", choices=["step", "fold", "align"])
+    ap.add_argument("--row", default="step", choices=["step", "fold", "align", "base"])
     ap.add_argument("--config", type=int, default=4, choices=[1, 2, 3, 4],
                     help="4: the 32-layer decode step (default); 1-3: the other serving configurations")
     ap.add_argument("--clocks-csv", default=None, help="also write the raw nvidia-smi samples of the timed region here")
@@ -1016,7 +1016,40 @@ def run_row(args, rank, world, local, pg):
         return (torch.randn(*shape, generator=gen, device=f"cuda:{local}") * std).to(torch.bfloat16)
 
     rc = 64
-    if args.row == "fold":
+    runner = None
+    flops = None
+    if args.row == "base":
+        # y = x W_base + the SALT delta for the 7 projections of one Llama-3.1-8B
+        # layer, the 512-token decode batch of the step (8 rank-64 centroids,
+        # rank-2 residuals drawn Zipf(1.1)); W_base as a linear layer stores it
+        from paper_2608_03579_gb300.runner import SaltRunner
+        w = wl.config4(seed=4, step=1, n_layers=1)
+        runner = SaltRunner(w, device=local, max_tokens=w.T)
+        runner.pin_centroids()
+        runner.load_slots()
+        runner.build(stream=stream)
+        torch.cuda.synchronize(local)
+        shapes = [(din, dout) for (_, din, dout) in w.layers]
+        n = len(shapes)
+        T = w.T
+        W = [randn(b, a, std=a ** -0.5) for (a, b) in shapes]
+        X = [randn(T, a) for (a, _) in shapes]
+        Y = [torch.empty(T, b, dtype=torch.bfloat16, device=f"cuda:{local}") for (_, b) in shapes]
+        ctx = None
+        flops = float(sum(2.0 * T * a * b for a, b in shapes) + sum(w.algorithmic_flops(l) for l in range(n)))
+        alg = float(sum(a * b * 2 + T * a * 2 + T * b * 2 for a, b in shapes)
+                    + sum(w.algorithmic_bytes(l) - T * (a * 2 + b * 4) for l, (a, b) in enumerate(shapes)))
+
+        def one(k):
+            for l in range(n):
+                salt.salt_lora_apply_with_base(runner.ctx, runner.seg, l, X[l], W[l], salt.SALT_W_OUT_IN, Y[l], stream)
+
+        def step_pair():
+            one(0)
+            one(1)
+        metric, unit, what = ("base GEMM fused with the SALT delta, TFLOP/s (y = x W_base + delta, one layer)",
+                              "TFLOP/s", "llama8b_layer_base_plus_delta_512tok")
+    elif args.row == "fold":
         d_in = [a for a, _ in shapes]
         d_out = [b for _, b in shapes]
         ctx = salt.salt_ctx_create(d_in, d_out, 1, rc, 1, 1, 16, local)
@@ -1106,9 +1139,29 @@ def run_row(args, rank, world, local, pg):
     ms = max_over_ranks(pg, e0.elapsed_time(e1), local) / steps_done
     achieved = alg / (ms / 1000.0) / 1e9
     clocks = sampler.summary()
+    flags = salt.salt_get_device_error(runner.ctx, None) if runner is not None else 0
     if ctx is not None:
         salt.salt_ctx_destroy(ctx)
-    if rank == 0:
+    if runner is not None:
+        runner.close()
+    if rank == 0 and args.row == "base":
+        tflops = flops / (ms / 1000.0) / 1e12
+        peak_t = peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"])
+        print(json.dumps({
+            "metric": metric, "value": world * tflops, "unit": unit, "n_gpus": world, "steps": steps_done,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": what, "tokens": T, "projections": n, "w_layout": "[d_out][d_in]",
+                       "flops_per_step": flops, "algorithmic_bytes_per_step": alg,
+                       "l2": "inputs larger than L2 (218 MB of base weights per layer)",
+                       "launch": "CUDA graph of two steps (per projection: a shrink-only apply, then the fused GEMM)"},
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak_t, "unit": "TFLOP/s",
+                         "frac": tflops / peak_t, "traffic": None,
+                         "hbm": {"achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                 "frac": achieved / peaks["hbm_gbs"]}},
+            "gpu_launches": steps_done * 2 * n, "valid": flags == 0,
+            "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")}}), flush=True)
+    elif rank == 0:
         launches = n if args.row == "fold" else 2 * ((n + 255) // 256)
         print(json.dumps({
             "metric": metric, "value": world * achieved, "unit": unit, "n_gpus": world, "steps": steps_done,
