@@ -232,6 +232,30 @@ salt_status salt_centroid_fold(salt_ctx *ctx, int32_t domain, int32_t layer, flo
                                int32_t layout, salt_stream_t stream);
 
 /*
+ * A fold plan: salt_centroid_fold over many weights in ONE launch (the
+ * same Section: when a node starts, a centroid is merged into every weight
+ * it adapts).  layers[i] and W[i] (i < n) name weight i as in
+ * salt_centroid_fold, all in `layout`; a layer may appear more than once
+ * with different weights, but no two weights may overlap in memory
+ * (SALT_ERR_INVALID_ARG).  The plan keeps the weights' addresses and the
+ * domain's pinned factors in device memory: the weights must stay allocated,
+ * and the centroid pinned, while the plan lives.  Host-side checks and one
+ * synchronous table upload; destroy the plan before its context.
+ */
+typedef struct salt_fold_plan salt_fold_plan;
+salt_status salt_fold_plan_create(salt_ctx *ctx, int32_t domain, int32_t n, const int32_t *layers,
+                                  void *const *W, int32_t layout, salt_fold_plan **out);
+/*
+ * W_i += gamma * s_c(domain) * A_c(layer_i) B_c(layer_i) for every weight
+ * of the plan, each element rounded once as in salt_centroid_fold (the
+ * results are bit-identical to n salt_centroid_fold calls).  One kernel,
+ * asynchronous on `stream`.  SALT_ERR_RANK when the domain was re-pinned
+ * with another rank after the plan was made.
+ */
+salt_status salt_fold_plan_run(salt_fold_plan *plan, float gamma, salt_stream_t stream);
+void salt_fold_plan_destroy(salt_fold_plan *plan);
+
+/*
  * Page-locked host memory for residual blobs, backed by transparent huge
  * pages where the kernel offers them (anonymous mapping rounded up to the
  * huge-page size, madvise(MADV_HUGEPAGE), every page touched, then

@@ -193,6 +193,14 @@ size_t apply_smem_bytes();
 // SALT_DEVERR_TIMEOUT in *err.
 cudaError_t launch_fold(const uint16_t *P, const uint16_t *Q, uint16_t *W, int Mdim, int Ndim, int rc, float scale,
                         uint32_t *err, cudaStream_t stream);
+// A fold plan's table: one record of fold_record_bytes() per weight (the
+// weight's TMA maps, P, its first item in the launch), written on the host
+// and copied to device memory; *n_items gets the weight's item count.
+size_t fold_record_bytes();
+cudaError_t fold_record(void *rec, const uint16_t *P, const uint16_t *Q, uint16_t *W, int Mdim, int Ndim, int rc,
+                        int64_t item0, int64_t *n_items);
+// Every weight of a device table of n records (items in all) in one launch.
+cudaError_t launch_fold_table(const void *table, int n, int64_t items, float scale, uint32_t *err, cudaStream_t stream);
 // salt_align_loss on the current device.
 salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
                            cudaStream_t stream);

@@ -583,6 +583,95 @@ salt_status salt_centroid_fold(salt_ctx *ctx, int32_t domain, int32_t layer, flo
     return SALT_OK;
 }
 
+struct salt_fold_plan {
+    salt_ctx *ctx = nullptr;
+    int32_t domain = 0, rc = 0, n = 0;
+    int64_t items = 0;
+    void *table = nullptr;  // device: n fold records
+};
+
+salt_status salt_fold_plan_create(salt_ctx *ctx, int32_t domain, int32_t n, const int32_t *layers, void *const *W,
+                                  int32_t layout, salt_fold_plan **out)
+{
+    if (!ctx || !out) return SALT_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (domain < 0 || domain >= ctx->n_domains)
+        return fail(ctx, SALT_ERR_DOMAIN_RANGE, "domain %d outside [0, %d)", domain, ctx->n_domains);
+    if (ctx->dom_rc[domain] == 0) return fail(ctx, SALT_ERR_DOMAIN_NOT_PINNED, "domain %d has no pinned centroid", domain);
+    if (n < 1 || !layers || !W) return fail(ctx, SALT_ERR_INVALID_ARG, "a fold plan needs n >= 1 layers and weights");
+    if (layout != SALT_W_IN_OUT && layout != SALT_W_OUT_IN) return fail(ctx, SALT_ERR_INVALID_ARG, "unknown layout %d", layout);
+    std::vector<std::pair<uintptr_t, uintptr_t>> spans;
+    for (int i = 0; i < n; ++i) {
+        const int l = layers[i];
+        if (l < 0 || l >= ctx->n_layers) return fail(ctx, SALT_ERR_LAYER_RANGE, "layer %d outside [0, %d)", l, ctx->n_layers);
+        if (!W[i]) return fail(ctx, SALT_ERR_INVALID_ARG, "null weight %d", i);
+        if (reinterpret_cast<uintptr_t>(W[i]) & 15u) return fail(ctx, SALT_ERR_ALIGN, "weight %d not 16-byte aligned", i);
+        const uintptr_t a = reinterpret_cast<uintptr_t>(W[i]);
+        spans.push_back({a, a + (uintptr_t)ctx->d_in[l] * ctx->d_out[l] * 2});
+    }
+    // the weights are updated in place by one launch: none may overlap another
+    std::sort(spans.begin(), spans.end());
+    for (size_t i = 1; i < spans.size(); ++i)
+        if (spans[i].first < spans[i - 1].second) return fail(ctx, SALT_ERR_INVALID_ARG, "weights of a fold plan overlap");
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    const int rc = ctx->dom_rc[domain];
+    const size_t rb = fold_record_bytes();
+    std::vector<uint8_t> host((size_t)n * rb);
+    int64_t items = 0;
+    for (int i = 0; i < n; ++i) {
+        const int l = layers[i];
+        const int din = ctx->d_in[l], dout = ctx->d_out[l];
+        const uint16_t *A = ctx->arenaA + ctx->a_off[l] + (int64_t)domain * ctx->rc_max * din;
+        const uint16_t *B = ctx->arenaB + ctx->b_off[l] + (int64_t)domain * ctx->rc_max * dout;
+        uint16_t *w = static_cast<uint16_t *>(W[i]);
+        int64_t k = 0;
+        const cudaError_t e = layout == SALT_W_IN_OUT ? fold_record(host.data() + i * rb, A, B, w, din, dout, rc, items, &k)
+                                                      : fold_record(host.data() + i * rb, B, A, w, dout, din, rc, items, &k);
+        if (e != cudaSuccess) return fail(ctx, SALT_ERR_CUDA, "fold record %d: %s", i, cudaGetErrorString(e));
+        items += k;
+    }
+    salt_fold_plan *pl = new (std::nothrow) salt_fold_plan;
+    if (!pl) return fail(ctx, SALT_ERR_OOM, "fold plan allocation failed");
+    if (cudaMalloc(&pl->table, host.size()) != cudaSuccess) {
+        delete pl;
+        return fail(ctx, SALT_ERR_OOM, "fold plan table allocation failed");
+    }
+    if (cudaMemcpy(pl->table, host.data(), host.size(), cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaFree(pl->table);
+        delete pl;
+        return fail(ctx, SALT_ERR_CUDA, "fold plan table copy failed");
+    }
+    pl->ctx = ctx;
+    pl->domain = domain;
+    pl->rc = rc;
+    pl->n = n;
+    pl->items = items;
+    *out = pl;
+    return SALT_OK;
+}
+
+salt_status salt_fold_plan_run(salt_fold_plan *plan, float gamma, salt_stream_t stream)
+{
+    if (!plan || !plan->ctx) return SALT_ERR_INVALID_ARG;
+    salt_ctx *ctx = plan->ctx;
+    if (ctx->dom_rc[plan->domain] != plan->rc)
+        return fail(ctx, SALT_ERR_RANK, "domain %d was re-pinned with rank %d after the plan was made (rank %d)", plan->domain,
+                    ctx->dom_rc[plan->domain], plan->rc);
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    const float scale = gamma * ctx->dom_sc[plan->domain];
+    CUDA_OR_FAIL(ctx, launch_fold_table(plan->table, plan->n, plan->items, scale, ctx->err_dev,
+                                        static_cast<cudaStream_t>(stream)));
+    return SALT_OK;
+}
+
+void salt_fold_plan_destroy(salt_fold_plan *plan)
+{
+    if (!plan) return;
+    if (plan->ctx) set_device(plan->ctx);
+    if (plan->table) cudaFree(plan->table);
+    delete plan;
+}
+
 salt_status salt_align_loss(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
                             salt_stream_t stream)
 {

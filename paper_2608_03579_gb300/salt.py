@@ -102,6 +102,9 @@ _SIGS = {
     "salt_host_pipe_wait": (ctypes.c_int, [_vp, _vp]),
     "salt_guard_check": (ctypes.c_int, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
     "salt_lora_apply_with_base": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp]),
+    "salt_fold_plan_create": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _i32, ctypes.POINTER(_vp)]),
+    "salt_fold_plan_run": (ctypes.c_int, [_vp, _f32, _vp]),
+    "salt_fold_plan_destroy": (None, [_vp]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -203,6 +206,36 @@ def salt_centroid_fold(ctx, domain: int, layer: int, gamma: float, W, layout: in
                        stream=None) -> None:
     """W += gamma * s_c(domain) * A_c B_c in place (W a CUDA bf16 tensor)."""
     _check(_lib.salt_centroid_fold(ctx, domain, layer, float(gamma), _ptr(W), layout, _stream(stream)), ctx)
+
+
+class FoldPlan:
+    """A salt_fold_plan handle; keeps the weight tensors alive with it."""
+
+    def __init__(self, ctx, handle, weights):
+        self.ctx, self.handle, self._weights = ctx, handle, weights
+
+
+def salt_fold_plan_create(ctx, domain: int, layers, weights, layout: int = SALT_W_IN_OUT) -> FoldPlan:
+    """One launch that folds domain's centroid into every weight (CUDA bf16
+    tensors) of `weights`, weights[i] being layer layers[i]'s."""
+    n = len(layers)
+    if len(weights) != n:
+        raise ValueError("one weight per layer")
+    ls = (ctypes.c_int32 * max(1, n))(*[int(l) for l in layers])
+    ws = (_vp * max(1, n))(*[_ptr(w) for w in weights])
+    h = _vp()
+    _check(_lib.salt_fold_plan_create(ctx, int(domain), n, ls, ws, int(layout), ctypes.byref(h)), ctx)
+    return FoldPlan(ctx, h, list(weights))
+
+
+def salt_fold_plan_run(plan: FoldPlan, gamma: float, stream=None) -> None:
+    _check(_lib.salt_fold_plan_run(plan.handle, float(gamma), _stream(stream)), plan.ctx)
+
+
+def salt_fold_plan_destroy(plan: FoldPlan) -> None:
+    if plan is not None and plan.handle:
+        _lib.salt_fold_plan_destroy(plan.handle)
+        plan.handle = None
 
 
 def salt_align_pairs(pairs):
