@@ -1165,7 +1165,7 @@ def run_row(args, rank, world, local, pg):
             "gpu_launches": steps_done * 2 * n, "valid": flags == 0,
             "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")}}), flush=True)
     elif rank == 0:
-        launches = 1 if args.row == "fold" else 2 * ((n + 255) // 256)
+        launches = 1 if args.row == "fold" else (n + 255) // 256
         print(json.dumps({
             "metric": metric, "value": world * achieved, "unit": unit, "n_gpus": world, "steps": steps_done,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",

@@ -480,7 +480,8 @@ salt_status salt_host_pipe_wait(salt_host_pipe *pipe, salt_stream_t stream);
  * factors F_in = [At ; At_c] ([r + rc][d_in]) and F_out = [B ; B_c], the
  * trace and both squared norms are sums over blocks of G_in o G_out, where
  * G = F F^T are (r + rc)^2 Gram matrices contracted on the tensor cores
- * (bf16 operands, fp32 accumulation) and combined in fp64.  The paper's
+ * (bf16 operands, fp32 accumulation) and combined in fp32 in a fixed
+ * order (the result does not depend on timing).  The paper's
  * eps is 1e-8.  pairs is a host array; its factor pointers are device bf16
  * arrays, rows contiguous, 16-byte aligned; 1 <= r, 1 <= rc,
  * r + rc <= SALT_MAX_ALIGN_RANK, d_in and d_out positive multiples of 8.

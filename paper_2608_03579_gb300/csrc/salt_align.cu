@@ -16,14 +16,16 @@
 // 64-column chunks of F stream through a cp.async ring into a 128-byte-
 // swizzled K-major tile that is both operands of tcgen05.mma
 // (D[128 x S] += F_chunk F_chunk^T, fp32 in tensor memory); the unit writes
-// its S x S partial.  align_combine_kernel: COMBINE_CTAS CTAs per pair, each
-// over a slice of the S x S entries, sum the partials of each side over the
-// splits in split order and form the slice's three block sums of
-// G_in o G_out (fp32: this part's fp64 rate is a small fraction of its fp32
-// rate, and the error added is far below the Gram entries' own fp32
-// accumulation error); the last CTA of a pair to finish (a counter) adds the
-// slices' sums in slice order in fp64 and writes the loss, so the result
-// does not depend on timing.
+// its S x S partial, then counts itself done for its pair.  The unit that
+// completes a pair (the last of its units to finish) combines it in the same
+// launch: its 128 threads sum each side's partials over the splits in split
+// order and form the three block sums of G_in o G_out, each thread over a
+// fixed set of entries, then a fixed shuffle tree and the four warps in
+// order, so the result does not depend on which unit finished last.  The
+// sums are fp32: this GPU's fp64 rate is a small fraction of its fp32 rate
+// (a dependent fp64 chain cost microseconds at the end of the launch), and
+// the rounding error added is far below the Gram entries' own fp32
+// accumulation error over d columns.
 #include "salt_async.cuh"
 #include "salt_internal.cuh"
 #include "salt_tcgen05.cuh"
@@ -41,8 +43,6 @@ constexpr int ALIGN_STAGE_BYTES = 128 * 128;     // <= 128 stacked rows x 64 col
 constexpr int ALIGN_SMEM = 1024 + ALIGN_STAGES * ALIGN_STAGE_BYTES;
 constexpr int ALIGN_MAX_PAIRS = 256;             // pairs per launch (the parameter block stays < 32 KB)
 constexpr int ALIGN_PART = 128 * 128;            // floats per unit partial (row pitch S)
-constexpr int COMBINE_THREADS = 256;
-constexpr int COMBINE_CTAS = 8;                  // CTAs per pair in the combine
 constexpr int KS_CAP = 16;                       // K-splits of one side at most
 static_assert(SALT_MAX_ALIGN_RANK <= 128, "a stack is the 128-row UMMA operand");
 
@@ -62,8 +62,7 @@ struct AlignParams {
     int32_t n_pairs;
     int32_t unit_start[2 * ALIGN_MAX_PAIRS + 1];  // first unit of (pair, side), then the total
     float *part;                                  // [units][ALIGN_PART]
-    double *sums;                                 // [pairs][COMBINE_CTAS][3]
-    uint32_t *done;                               // [pairs]: combine CTAs finished (zeroed)
+    uint32_t *done;                               // [pairs]: units finished (zeroed)
     float *loss;
     float *cosine;                                // may be null
     float eps;
@@ -163,7 +162,9 @@ __global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_
         }
     tc_fence_after();
 
-    // D rows (tensor-memory lanes) = stack rows, columns = stack rows
+    // D rows (tensor-memory lanes) = stack rows, columns = stack rows.  D
+    // is symmetric: thread `row` writes D's row as column `row`, so a
+    // warp's stores of one column are contiguous.
     float *out = p.part + (int64_t)unit * ALIGN_PART;
     const int row = warp * 32 + lane;
     for (int g = 0; g < n_pad / 16; ++g) {
@@ -173,90 +174,99 @@ __global__ void __launch_bounds__(ALIGN_THREADS) align_gram_kernel(const __grid_
         if (row < S) {
 #pragma unroll
             for (int e = 0; e < 16; ++e)
-                if (g * 16 + e < S) out[row * S + g * 16 + e] = __uint_as_float(v[e]);
+                if (g * 16 + e < S) __stcg(out + (g * 16 + e) * S + row, __uint_as_float(v[e]));
         }
     }
     if (!ok_all) atomicOr(p.err, SALT_DEVERR_TIMEOUT);
+    __threadfence();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 128);
-}
 
-__device__ float block_sum(float v, float *red)
-{
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    float t = 0.f;
-    if (threadIdx.x == 0)
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
-    __syncthreads();
-    return t;  // valid in thread 0
-}
-
-// sum over the K-splits of one Gram entry, split order; the loads are issued together
-__device__ __forceinline__ float split_sum(const float *part, int u0, int ks, int idx)
-{
-    float v[KS_CAP];
-#pragma unroll
-    for (int s = 0; s < KS_CAP; ++s) v[s] = s < ks ? __ldcg(part + (int64_t)(u0 + s) * ALIGN_PART + idx) : 0.f;
-    float acc = v[0];
-#pragma unroll
-    for (int s = 1; s < KS_CAP; ++s) acc += v[s];
-    return acc;
-}
-
-__global__ void __launch_bounds__(COMBINE_THREADS) align_combine_kernel(const __grid_constant__ AlignParams p)
-{
-    __shared__ float red[COMBINE_THREADS / 32];
-    __shared__ bool last;
-    const int pi = blockIdx.x / COMBINE_CTAS, slice = blockIdx.x - pi * COMBINE_CTAS;
-    const AlignPairP &pr = p.pair[pi];
-    const int r = pr.r, S = pr.r + pr.rc;
+    // ------------------------------------------------ the pair's combine
+    __shared__ int last;
+    __shared__ float red[3][ALIGN_THREADS / 32];
+    const int pi = ps >> 1;
+    const AlignPairP &pq = p.pair[pi];
     const int u_in = p.unit_start[2 * pi], u_out = p.unit_start[2 * pi + 1];
-    const int ks_in = pr.side[0].ks, ks_out = pr.side[1].ks;
-    const int i0 = S * S * slice / COMBINE_CTAS, i1 = S * S * (slice + 1) / COMBINE_CTAS;
-    float num = 0.f, na = 0.f, nc = 0.f;
-    for (int idx = i0 + threadIdx.x; idx < i1; idx += COMBINE_THREADS) {
-        const int i = idx / S, j = idx - i * S;
-        if (i >= r && j < r) continue;  // the lower cross block mirrors the upper one
-        const float gi = split_sum(p.part, u_in, ks_in, idx);
-        const float go = split_sum(p.part, u_out, ks_out, idx);
-        const float prod = gi * go;
-        if (i < r && j < r) na += prod;
-        else if (i >= r) nc += prod;
-        else num += prod;
-    }
-    num = block_sum(num, red);
-    na = block_sum(na, red);
-    nc = block_sum(nc, red);
-    if (threadIdx.x == 0) {
-        double *o = p.sums + ((int64_t)pi * COMBINE_CTAS + slice) * 3;
-        o[0] = num;
-        o[1] = na;
-        o[2] = nc;
+    const int ks_in = pq.side[0].ks, ks_out = pq.side[1].ks;
+    if (tid == 0) {
+        last = atomicAdd(p.done + pi, 1u) == (uint32_t)(ks_in + ks_out) - 1u;
         __threadfence();
-        last = atomicAdd(p.done + pi, 1u) == COMBINE_CTAS - 1;
     }
     __syncthreads();
-    if (last && threadIdx.x == 0) {
-        __threadfence();
-        double dnum = 0.0, dna = 0.0, dnc = 0.0;
-        for (int c = 0; c < COMBINE_CTAS; ++c) {
-            const volatile double *q = p.sums + ((int64_t)pi * COMBINE_CTAS + c) * 3;
-            dnum += q[0];
-            dna += q[1];
-            dnc += q[2];
+    if (!last) return;
+    // every partial of the pair is written.  Thread t takes the float4 of
+    // entries t, t + 128, ... (the partials' pitch of 16384 floats keeps the
+    // last float4 in bounds; entries past S * S are skipped); up to four
+    // splits of a side are loaded together before they are added.
+    const int SS = S * S, n4 = (SS + 3) / 4;
+    const float4 *pin = reinterpret_cast<const float4 *>(p.part + (int64_t)u_in * ALIGN_PART);
+    const float4 *pout = reinterpret_cast<const float4 *>(p.part + (int64_t)u_out * ALIGN_PART);
+    constexpr int U4 = ALIGN_PART / 4;
+    float num = 0.f, na = 0.f, nc = 0.f;
+    for (int b4 = tid; b4 < n4; b4 += ALIGN_THREADS) {
+        float gi[4] = {0.f, 0.f, 0.f, 0.f}, go[4] = {0.f, 0.f, 0.f, 0.f};
+        auto add_side = [&](const float4 *base, int ks, float (&acc)[4]) {
+            for (int k0 = 0; k0 < ks; k0 += 4) {
+                float4 x[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    x[k] = k0 + k < ks ? __ldcg(base + (int64_t)(k0 + k) * U4 + b4) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    acc[0] += x[k].x;
+                    acc[1] += x[k].y;
+                    acc[2] += x[k].z;
+                    acc[3] += x[k].w;
+                }
+            }
+        };
+        add_side(pin, ks_in, gi);
+        add_side(pout, ks_out, go);
+        const int idx0 = b4 * 4;
+        int i = idx0 / S, j = idx0 - i * S;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            // the lower cross block mirrors the upper one
+            if (idx0 + e < SS && !(i >= r && j < r)) {
+                const float prod = gi[e] * go[e];
+                if (i < r && j < r) na += prod;
+                else if (i >= r) nc += prod;
+                else num += prod;
+            }
+            if (++j == S) {
+                j = 0;
+                ++i;
+            }
         }
-        const double tr = (double)pr.s * (double)pr.s_c * dnum;
-        const double n_dw = fabs((double)pr.s) * sqrt(fmax(dna, 0.0));
-        const double n_wb = fabs((double)pr.s_c) * sqrt(fmax(dnc, 0.0));
-        double cosv = tr / (n_dw * n_wb + (double)p.eps);
-        if (*reinterpret_cast<volatile uint32_t *>(p.err) != 0u) cosv = __longlong_as_double(0x7ff8000000000000ll);
-        p.loss[pi] = (float)(1.0 - cosv);
-        if (p.cosine) p.cosine[pi] = (float)cosv;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        num += __shfl_xor_sync(0xffffffffu, num, o);
+        na += __shfl_xor_sync(0xffffffffu, na, o);
+        nc += __shfl_xor_sync(0xffffffffu, nc, o);
+    }
+    if (lane == 0) {
+        red[0][warp] = num;
+        red[1][warp] = na;
+        red[2][warp] = nc;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        float snum = 0.f, sna = 0.f, snc = 0.f;
+        for (int w = 0; w < ALIGN_THREADS / 32; ++w) {
+            snum += red[0][w];
+            sna += red[1][w];
+            snc += red[2][w];
+        }
+        const float tr = pq.s * pq.s_c * snum;
+        const float n_dw = fabsf(pq.s) * sqrtf(fmaxf(sna, 0.f));
+        const float n_wb = fabsf(pq.s_c) * sqrtf(fmaxf(snc, 0.f));
+        float cosv = tr / (n_dw * n_wb + p.eps);
+        if (*reinterpret_cast<volatile uint32_t *>(p.err) != 0u) cosv = __int_as_float(0x7fc00000);
+        p.loss[pi] = 1.f - cosv;
+        if (p.cosine) p.cosine[pi] = cosv;
     }
 }
 
@@ -340,12 +350,11 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
             u += ks[2 * i + 1];
         }
         p.unit_start[2 * m] = u;
-        // scratch: the error word and the pairs' counters (zeroed), the
-        // combine's slice sums, then the partials
+        // scratch: the error word and the pairs' counters (zeroed), then
+        // the partials
         const size_t head = 256 + (size_t)ALIGN_MAX_PAIRS * 4;
-        const size_t sums = (size_t)ALIGN_MAX_PAIRS * COMBINE_CTAS * 3 * sizeof(double);
         void *ws = nullptr;
-        const size_t bytes = head + sums + (size_t)u * ALIGN_PART * sizeof(float);
+        const size_t bytes = head + (size_t)u * ALIGN_PART * sizeof(float);
         if (cudaMallocAsync(&ws, bytes, stream) != cudaSuccess) {
             cudaGetLastError();
             return SALT_ERR_OOM;
@@ -353,15 +362,10 @@ salt_status align_loss_run(int32_t n, const salt_align_pair *pairs, float eps, f
         uint8_t *w8 = static_cast<uint8_t *>(ws);
         p.err = reinterpret_cast<uint32_t *>(w8);
         p.done = reinterpret_cast<uint32_t *>(w8 + 256);
-        p.sums = reinterpret_cast<double *>(w8 + head);
-        p.part = reinterpret_cast<float *>(w8 + head + sums);
+        p.part = reinterpret_cast<float *>(w8 + head);
         cudaError_t e = cudaMemsetAsync(ws, 0, head, stream);
         if (e == cudaSuccess) {
             align_gram_kernel<<<u, ALIGN_THREADS, ALIGN_SMEM, stream>>>(p);
-            e = cudaGetLastError();
-        }
-        if (e == cudaSuccess) {
-            align_combine_kernel<<<m * COMBINE_CTAS, COMBINE_THREADS, 0, stream>>>(p);
             e = cudaGetLastError();
         }
         cudaError_t f = cudaFreeAsync(ws, stream);

@@ -4,8 +4,10 @@ fp64 oracle.
 Tolerance.  Each Gram entry G_ij = sum_t F_it F_jt is an fp32 sum of d exact
 products (a product of two bf16 is exact in fp32), so its error is at most
 about d u sum_t |F_it F_jt| with u = 2^-24; the test allows 4 d u.  The
-trace and the squared norms are block sums of G_in o G_out (formed in fp64),
-so their errors are bounded by the same sums with |G| and the entry bounds;
+trace and the squared norms are block sums of G_in o G_out, so their errors
+are bounded by the same sums with |G| and the entry bounds, plus the fp32
+rounding of the products and of the sums themselves (fixed order, at most 64
+additions deep: 66 u times the block's sum of |G_in o G_out|);
 the cosine's error follows to first order.  The bound is computed from the
 factors of each case, with a floor of 1e-6 (float output)."""
 import numpy as np
@@ -25,7 +27,7 @@ def _bound(wl, At, B, Atc, Bc, s, s_c, cos_ref):
     Gi, Go = Fi @ Fi.T, Fo @ Fo.T
     Ei = 4 * Fi.shape[1] * 2.0 ** -24 * (np.abs(Fi) @ np.abs(Fi).T)
     Eo = 4 * Fo.shape[1] * 2.0 ** -24 * (np.abs(Fo) @ np.abs(Fo).T)
-    E = Ei * np.abs(Go) + np.abs(Gi) * Eo + Ei * Eo
+    E = Ei * np.abs(Go) + np.abs(Gi) * Eo + Ei * Eo + 66 * 2.0 ** -24 * np.abs(Gi * Go)
     num_e = E[:r, r:].sum()
     na, nc = (Gi * Go)[:r, :r].sum(), (Gi * Go)[r:, r:].sum()
     na_e, nc_e = E[:r, :r].sum(), E[r:, r:].sum()
