@@ -179,6 +179,50 @@ __device__ void item_at(const int32_t *blk, int n_blk, int nu, int64_t total, in
     }
 }
 
+// With no more (row block, projection) pairs than CTAs, each pair gets its
+// own contiguous CTAs: one each, plus a share of the rest proportional to
+// the pair's expand cost (its 64-column items times the block's weight), so
+// that no CTA expands two pairs (a second run costs a table phase, a V wait
+// and a refill of the ring: measured at 3-5 us, enough to make those CTAs
+// the launch's tail).  The pair's items are split evenly over its CTAs.
+// CTA g gets block *b and items [*u0, *u1) (absolute unit indices, u1 <= nu).
+// Whole warp.
+__device__ void pair_range(const ApplyParams &p, int n_blk, int nu, int g, int lane, int &b, int &u0, int &u1)
+{
+    const int G = gridDim.x, np = p.n_proj;
+    const int n_bp = n_blk * np;
+    const int64_t R = G - n_bp;  // CTAs beyond one per pair
+    const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
+    // first CTA of pair j = (bb, pi): j + floor(C_j * R / total), C_j its cost prefix
+    auto first_cta = [&](int bb, int pi) -> int64_t {
+        if (bb >= n_blk) return G;
+        const int64_t wbeg = bb ? blk_wend(p.blk, bb - 1) : 0;
+        const int64_t w = blk_wend(p.blk, bb) - wbeg;
+        const int64_t C = (int64_t)nu * wbeg + (int64_t)p.n_unit_prefix[pi] * w;
+        return (int64_t)bb * np + pi + (total > 0 ? C * R / total : 0);
+    };
+    // the last block whose first pair starts at or before g
+    int lo = 0, hi = n_blk;  // answer in [lo, hi)
+    while (hi - lo > 1) {
+        const int step = (hi - lo + 31) >> 5;
+        const int i = lo + lane * step;
+        const bool le = i < hi && first_cta(i, 0) <= g;
+        const unsigned m = __ballot_sync(0xffffffffu, le);
+        const int last = 31 - __clz(m);  // lane 0 always holds (first_cta(lo, 0) <= g)
+        lo = lo + last * step;
+        hi = min(hi, lo + step);
+    }
+    b = lo;
+    int pi = 0;
+    while (pi + 1 < np && first_cta(b, pi + 1) <= g) ++pi;
+    const int64_t f0 = first_cta(b, pi);
+    const int64_t f1 = pi + 1 < np ? first_cta(b, pi + 1) : first_cta(b + 1, 0);
+    const int64_t c = f1 - f0, k = g - f0;
+    const int base = p.n_unit_prefix[pi], U = p.n_unit_prefix[pi + 1] - base;
+    u0 = base + (int)(k * U / c);
+    u1 = base + (int)((k + 1) * U / c);
+}
+
 constexpr int MAX_PIECES = (TM * 8 + APPLY_THREADS - 1) / APPLY_THREADS;  // 16-byte pieces per thread and chunk
 constexpr int N_QUADS = APPLY_THREADS / 128;  // full groups of 4 warps (one per TMEM lane quarter)
 constexpr int EPI_WARP0 = PRODUCER_WARPS + 1;  // first epilogue warp
@@ -415,9 +459,16 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     // tables, off the critical path.
     bool have_range = false;
     auto find_range = [&](int e) {
-        const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
         int b = n_blk, u = 0;  // no expand items when only the V tiles are wanted
-        if (!p.shrink_only) item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + e) / gridDim.x, lane, b, u);
+        if (p.shrink_only) {
+        } else if (n_bp <= (int)gridDim.x) {
+            int u0, u1;
+            pair_range(p, n_blk, nu, blockIdx.x, lane, b, u0, u1);
+            u = e ? u1 : u0;
+        } else {
+            const int64_t total = (int64_t)nu * blk_wend(p.blk, n_blk - 1);
+            item_at(p.blk, n_blk, nu, total, total * (blockIdx.x + e) / gridDim.x, lane, b, u);
+        }
         if (lane == 0) {
             info.range[2 * e] = b;
             info.range[2 * e + 1] = u;
