@@ -326,7 +326,12 @@ salt_status salt_build_segments(salt_ctx *ctx, salt_segments *seg,
  * scale s_c(d) * gamma[g]; a token without a centroid ignores its bin.
  * Tokens are sorted stably by (domain, bin, slot), -1 first; domain runs
  * become runs of equal (domain, bin) and user runs runs of equal (domain,
- * bin, slot) (their bins: salt_segments_export_gamma).  A bin outside the
+ * bin, slot) (their bins: salt_segments_export_gamma).  The row blocks of
+ * the apply kernels are cut from the same tokens ordered by (domain, slot)
+ * instead (gamma multiplies each token's centroid term), so a user whose
+ * tokens fall in several bins takes one set of residual rows in a block;
+ * the blocks salt_segments_export reports index that order, which spans the
+ * same positions as the grouped order for every domain.  A bin outside the
  * range is SALT_ERR_GAMMA_RANGE for host ids, SALT_DEVERR_GAMMA_RANGE (and
  * bin -1) for device ids.  Otherwise as salt_build_segments, which is this
  * call with every bin -1.

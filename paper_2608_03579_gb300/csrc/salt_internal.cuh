@@ -59,6 +59,16 @@ struct SegDev {
     float *tok_sc;         // [max_tokens]
     // per row block: residual rows of the factor stack, res_code(slot, rank, k)
     int32_t *blk_res;      // [max_tokens * S_MAX]
+    // The apply order: the tokens stably sorted by (domain, slot), gamma bin
+    // after the slot.  Row blocks, blk_res and the per-token tables above
+    // (sorted_slot, tok_*) index this order.  Without gamma bins it is the
+    // grouped order (perm); with them a user's tokens in several bins are
+    // one run here, so they share one set of residual rows in a block.
+    int32_t *aperm;        // [max_tokens] token index in apply order
+    int32_t *a_dptr;       // [max_tokens + 1] domain runs of the apply order (gamma builds)
+    int32_t *a_ddom;       // [max_tokens]
+    int32_t *a_uptr;       // [max_tokens + 1] (domain, slot) runs of the apply order (gamma builds)
+    int32_t *a_udom;       // [max_tokens]
 };
 
 // Code of one residual row of a factor stack: row k of the rank-`rank`

@@ -801,7 +801,8 @@ salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)
               alloc(&seg->d.blk, (size_t)BLK_INTS * n) && alloc(&seg->d.counts, 4) && alloc(&seg->d.tok_uoff, n) &&
               alloc(&seg->d.tok_urank, n) && alloc(reinterpret_cast<int32_t **>(&seg->d.tok_su), n) &&
               alloc(reinterpret_cast<int32_t **>(&seg->d.tok_sc), n) &&
-              alloc(&seg->d.blk_res, (size_t)n * S_MAX);
+              alloc(&seg->d.blk_res, (size_t)n * S_MAX) && alloc(&seg->d.aperm, n) && alloc(&seg->d.a_dptr, n + 1) &&
+              alloc(&seg->d.a_ddom, n) && alloc(&seg->d.a_uptr, n + 1) && alloc(&seg->d.a_udom, n);
     seg->work.blk_cap = block_bound_loose(ctx, n);
     seg->work.max_group = SALT_MAX_GROUP;
     seg->work.part_cap = PART_CAP;
@@ -848,7 +849,7 @@ void salt_segments_destroy(salt_segments *seg)
                        seg->d.useg_slot, seg->d.blk, seg->d.counts,
                        seg->d.tok_uoff, seg->d.tok_urank, reinterpret_cast<int32_t *>(seg->d.tok_su),
                        reinterpret_cast<int32_t *>(seg->d.tok_sc),
-                       seg->d.blk_res};
+                       seg->d.blk_res, seg->d.aperm, seg->d.a_dptr, seg->d.a_ddom, seg->d.a_uptr, seg->d.a_udom};
     for (int32_t *p : arrs) cudaFree(p);
     guarded_free(seg->work.vext);
     guarded_free(seg->work.part);
@@ -1078,7 +1079,7 @@ salt_status apply_grouped(salt_ctx *ctx, const salt_segments *seg_, int32_t n, c
     p.n_unit_prefix[n] = units;
     p.min_nk = 1 << 30;
     for (int i = 0; i < n; ++i) p.min_nk = std::min(p.min_nk, (p.proj[i].d_in + 63) / 64);
-    p.perm = seg->d.perm;
+    p.perm = seg->d.aperm;
     p.blk = seg->d.blk;
     p.counts = seg->d.counts;
     p.tok_uoff = seg->d.tok_uoff;
@@ -1134,7 +1135,7 @@ salt_status salt_lora_apply_with_base(salt_ctx *ctx, const salt_segments *seg_, 
     CUDA_OR_FAIL(ctx, encode_base_map(&bp.wmap, static_cast<const uint16_t *>(W), din, dout, layout));
     bp.x = static_cast<const uint16_t *>(x);
     bp.y = static_cast<uint16_t *>(y);
-    bp.perm = seg->d.perm;
+    bp.perm = seg->d.aperm;
     bp.blk = seg->d.blk;
     bp.counts = seg->d.counts;
     bp.blk_res = seg->d.blk_res;
@@ -1203,7 +1204,7 @@ salt_status salt_lora_apply_static(salt_ctx *ctx, const salt_segments *seg_, int
     p.n_unit_prefix[0] = 0;
     p.n_unit_prefix[1] = (pr.d_out + 63) / 64;
     p.min_nk = (pr.d_in + 63) / 64;
-    p.perm = seg->d.perm;
+    p.perm = seg->d.aperm;
     p.blk = seg->d.blk;
     p.counts = seg->d.counts;
     p.tok_uoff = seg->d.tok_uoff;

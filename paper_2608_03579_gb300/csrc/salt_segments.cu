@@ -82,6 +82,28 @@ __device__ __forceinline__ int upper_index(const int32_t *a, int lo, int hi, int
     return lo;
 }
 
+// Ascending bitonic sort of n (a power of two) keys in shared memory; the
+// whole block calls it.
+__device__ void bitonic_sort(uint64_t *keys, int n)
+{
+    for (int k = 2; k <= n; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = threadIdx.x; i < n; i += blockDim.x) {
+                int ixj = i ^ j;
+                if (ixj > i) {
+                    uint64_t a = keys[i], b = keys[ixj];
+                    bool up = (i & k) == 0;
+                    if ((a > b) == up) {
+                        keys[i] = b;
+                        keys[ixj] = a;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
 __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
 {
     extern __shared__ __align__(16) uint64_t keys[];
@@ -145,22 +167,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     __syncthreads();
 
     // 2. bitonic sort, ascending
-    for (int k = 2; k <= P2; k <<= 1) {
-        for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int i = tid; i < P2; i += nth) {
-                int ixj = i ^ j;
-                if (ixj > i) {
-                    uint64_t a = keys[i], b = keys[ixj];
-                    bool up = (i & k) == 0;
-                    if ((a > b) == up) {
-                        keys[i] = b;
-                        keys[ixj] = a;
-                    }
-                }
-            }
-            __syncthreads();
-        }
-    }
+    bitonic_sort(keys, P2);
 
     // 3. runs: count heads per contiguous chunk, scan, then write
     const int E = (T + nth - 1) / nth;
@@ -180,6 +187,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         uint64_t k = keys[i];
         int d = key_dom(k), gb = key_gb(k), s = key_slot(k);
         p.s.perm[i] = key_tok(k);
+        p.s.aperm[i] = key_tok(k);
         p.s.sorted_slot[i] = s;
         p.s.tok_sc[i] = d >= 0 ? p.dom_sc[d] * (gb >= 0 ? p.gamma[gb] : 1.f) : 0.f;
         bool dh = i == 0 || key_cent(k) != key_cent(keys[i - 1]);
@@ -203,23 +211,82 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         p.s.useg_ptr[n_useg] = T;
     }
     const bool skip0 = key_dom(keys[0]) == -1 && key_slot(keys[0]) == -1;
+    // The runs the row blocks are cut from: the grouped order's, unless the
+    // batch has gamma bins (below).
+    const int32_t *dptr = p.s.dseg_ptr, *ddom = p.s.dseg_dom, *uptr = p.s.useg_ptr, *udom = p.s.useg_dom;
+    int n_dr = n_dseg, n_ur = n_useg;
+    if (p.has_gbin) {
+        // 3'. The apply order: the same keys re-sorted by (domain, slot, bin,
+        //     token), so that a user's tokens in several bins form one run
+        //     and take one set of residual rows in a block (gamma is applied
+        //     per token).  Writes aperm and, in this order, sorted_slot,
+        //     tok_sc and the domain and (domain, slot) runs.
+        __syncthreads();  // every thread is done with the grouped order
+        for (int i = tid; i < P2; i += nth) {
+            const uint64_t k = keys[i];
+            if (k != ~0ull)
+                keys[i] = (key_cent(k) >> KEY_GB_BITS) << (KEY_CENT_SHIFT + KEY_GB_BITS) |
+                          (uint64_t)(key_slot(k) + 1) << (KEY_TOK_BITS + KEY_GB_BITS) |
+                          (uint64_t)(key_gb(k) + 1) << KEY_TOK_BITS | (uint64_t)key_tok(k);
+        }
+        __syncthreads();
+        bitonic_sort(keys, P2);
+        // fields of an apply-order key: domain + 1 | slot + 1 | bin + 1 | token
+        auto a_dom = [](uint64_t k) { return (int)(k >> (KEY_CENT_SHIFT + KEY_GB_BITS)) - 1; };
+        auto a_slot = [](uint64_t k) { return (int)((k >> (KEY_TOK_BITS + KEY_GB_BITS)) & KEY_SLOT_MASK) - 1; };
+        auto a_gb = [](uint64_t k) { return (int)((k >> KEY_TOK_BITS) & KEY_GB_MASK) - 1; };
+        auto a_user = [](uint64_t k) { return k >> (KEY_TOK_BITS + KEY_GB_BITS); };
+        int ad = 0, au = 0;
+        for (int i = lo; i < hi; ++i) {
+            const uint64_t k = keys[i];
+            ad += i == 0 || a_dom(k) != a_dom(keys[i - 1]);
+            au += i == 0 || a_user(k) != a_user(keys[i - 1]);
+        }
+        int oad = block_exclusive_scan(ad, &n_dr, warp_sums);
+        int oau = block_exclusive_scan(au, &n_ur, warp_sums);
+        for (int i = lo; i < hi; ++i) {
+            const uint64_t k = keys[i];
+            const int d = a_dom(k), gb = a_gb(k), sl = a_slot(k);
+            p.s.aperm[i] = key_tok(k);
+            p.s.sorted_slot[i] = sl;
+            p.s.tok_sc[i] = d >= 0 ? p.dom_sc[d] * (gb >= 0 ? p.gamma[gb] : 1.f) : 0.f;
+            if (i == 0 || a_dom(k) != a_dom(keys[i - 1])) {
+                p.s.a_dptr[oad] = i;
+                p.s.a_ddom[oad] = d;
+                ++oad;
+            }
+            if (i == 0 || a_user(k) != a_user(keys[i - 1])) {
+                p.s.a_uptr[oau] = i;
+                p.s.a_udom[oau] = d;
+                ++oau;
+            }
+        }
+        if (tid == 0) {
+            p.s.a_dptr[n_dr] = T;
+            p.s.a_uptr[n_ur] = T;
+        }
+        dptr = p.s.a_dptr;
+        ddom = p.s.a_ddom;
+        uptr = p.s.a_uptr;
+        udom = p.s.a_udom;
+    }
     __syncthreads();  // keys are dead from here; run arrays are visible block-wide
 
     // 4a. group heads over user runs; a group stays within one domain (the
     //     (domain, bin) runs of a domain are consecutive)
     int32_t *grp_first = reinterpret_cast<int32_t *>(keys);  // [n_groups]
-    const int Eu = (n_useg + nth - 1) / nth;
-    const int ulo = min(n_useg, tid * Eu), uhi = min(n_useg, ulo + Eu);
+    const int Eu = (n_ur + nth - 1) / nth;
+    const int ulo = min(n_ur, tid * Eu), uhi = min(n_ur, ulo + Eu);
     auto group_head = [&](int j) -> bool {
         if (j == 0) return true;
         if (skip0 && j == 1) return true;
-        int start = p.s.useg_ptr[j];
-        int dr = upper_index(p.s.dseg_ptr, 0, n_dseg, start);
-        const int d = p.s.dseg_dom[dr];
-        while (dr > 0 && p.s.dseg_dom[dr - 1] == d) --dr;  // at most SALT_MAX_GAMMA_BINS steps
-        int dstart = p.s.dseg_ptr[dr];
+        int start = uptr[j];
+        int dr = upper_index(dptr, 0, n_dr, start);
+        const int d = ddom[dr];
+        while (dr > 0 && ddom[dr - 1] == d) --dr;  // at most SALT_MAX_GAMMA_BINS steps
+        int dstart = dptr[dr];
         if (dstart == start) return true;  // first user run of a domain
-        int first = upper_index(p.s.useg_ptr, 0, n_useg, dstart);
+        int first = upper_index(uptr, 0, n_ur, dstart);
         int idx = j - first - ((skip0 && dr == 0) ? 1 : 0);
         return idx % p.umax == 0;
     };
@@ -235,8 +302,8 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
     const int Eg = (n_groups + nth - 1) / nth;
     const int glo = min(n_groups, tid * Eg), ghi = min(n_groups, glo + Eg);
     auto group_range = [&](int g, int *start, int *len) {
-        int a = p.s.useg_ptr[grp_first[g]];
-        int b = g + 1 < n_groups ? p.s.useg_ptr[grp_first[g + 1]] : T;
+        int a = uptr[grp_first[g]];
+        int b = g + 1 < n_groups ? uptr[grp_first[g + 1]] : T;
         *start = a;
         *len = (g == 0 && skip0) ? 0 : b - a;
     };
@@ -252,7 +319,7 @@ __global__ void __launch_bounds__(SEG_THREADS, 1) seg_build_kernel(SegParams p)
         int a, len;
         group_range(g, &a, &len);
         int q = (len + TM - 1) / TM;
-        int d = p.s.useg_dom[grp_first[g]];
+        int d = udom[grp_first[g]];
         const float sc = d >= 0 ? p.dom_sc[d] : 0.f;
         for (int b = 0; b < q; ++b) {
             int s0 = a + (int)(((int64_t)b * len) / q);
