@@ -327,7 +327,42 @@ __device__ void finish_split_unit(const ApplyParams &p, FusedInfo &info, const U
     // user's), in split order, staged in shared memory, then scaled, masked
     // and written as bf16 V rows
     constexpr int PC4 = PART_COLS / 4;
-    for (int idx = tid; idx < (r1 - r0) * PC4; idx += nthr) {
+    const int n_it = (r1 - r0) * PC4;
+    // (row, 4 columns) items of the slice; with up to 8 splits a thread
+    // takes two items at once, so all of its loads are in flight together
+    constexpr int KS_PAIR = 8;
+    for (int idx = tid; KS <= KS_PAIR && idx < n_it; idx += 2 * nthr) {
+        float4 v[2][KS_PAIR];
+        bool use[2];
+        const float *src[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int it = idx + h * nthr, rr = it / PC4, c4 = it - rr * PC4, t = r0 + rr;
+            use[h] = it < n_it && c4 * 4 < rc + info.urank[t];
+            src[h] = p.w.part + ((int64_t)g.pair * KS * TM + t) * PART_COLS + c4 * 4;
+#pragma unroll
+            for (int s2 = 0; s2 < KS_PAIR; ++s2) {
+                v[h][s2] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (use[h] && ((ne_mask >> s2) & 1))
+                    v[h][s2] = __ldcg(reinterpret_cast<const float4 *>(src[h] + (int64_t)s2 * (TM * PART_COLS)));
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            if (!use[h]) continue;
+            float4 acc = v[h][0];
+#pragma unroll
+            for (int s2 = 1; s2 < KS_PAIR; ++s2) {
+                acc.x += v[h][s2].x;
+                acc.y += v[h][s2].y;
+                acc.z += v[h][s2].z;
+                acc.w += v[h][s2].w;
+            }
+            const int it = idx + h * nthr, rr = it / PC4, c4 = it - rr * PC4;
+            *reinterpret_cast<float4 *>(Ps + rr * PART_COLS + c4 * 4) = acc;
+        }
+    }
+    for (int idx = tid; KS > KS_PAIR && idx < n_it; idx += nthr) {
         const int rr = idx / PC4, c4 = idx - rr * PC4, t = r0 + rr;
         if (c4 * 4 >= rc + info.urank[t]) continue;
         float4 v[KS_MAX];
@@ -400,8 +435,15 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     int KS = max(1, min(KS_MAX, (int)gridDim.x / n_bp));
     if (KS > 1 && (int64_t)n_bp * KS > p.w.part_cap) KS = max(1, p.w.part_cap / n_bp);
     const int n_units = n_bp * KS;
-    const int ua = (int)((int64_t)n_units * blockIdx.x / gridDim.x);
-    const int ub = (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
+    // With at most one unit per CTA the units go to the lowest CTA indices:
+    // the CTAs of a launch start in index order as the previous launch's
+    // CTAs leave their SMs, so the last ones to start (up to a few
+    // microseconds late) are the ones without a shrink unit, and no block
+    // waits for a late split.
+    const int ua = n_units <= (int)gridDim.x ? min((int)blockIdx.x, n_units)
+                                             : (int)((int64_t)n_units * blockIdx.x / gridDim.x);
+    const int ub = n_units <= (int)gridDim.x ? min((int)blockIdx.x + 1, n_units)
+                                             : (int)((int64_t)n_units * (blockIdx.x + 1) / gridDim.x);
 
     const uint32_t bb = smem_u32(&info.bbar[0]);
     auto full_bar = [&](int st) { return bb + 8u * st; };
@@ -454,9 +496,11 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     };
 
     // This CTA's share of the expand items: the first (e = 0) or end (e = 1)
-    // item of its cost range, into info.range; one warp each.  Searched by
-    // warps 0 and 1 while the other warps write the first shrink unit's
-    // tables, off the critical path.
+    // item of its range, into info.range; one warp each.  With split
+    // shrinks, searched by warps 0 and 1 when the shrink phase is over
+    // (while the block's splits are reduced), so that the first shrink
+    // unit's table phase does not wait for the search; with single splits,
+    // during that table phase.
     bool have_range = false;
     auto find_range = [&](int e) {
         int b = n_blk, u = 0;  // no expand items when only the V tiles are wanted
@@ -495,9 +539,10 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
             continue;
         }
         __syncthreads();  // the previous unit is done with info and the ring
-        // the token and factor tables (threads 64..191); meanwhile warps 0 and
-        // 1 find the CTA's expand items
-        if (!have_range && warp < 2) {
+        // the token and factor tables (threads 64..191); with single splits
+        // (the expand follows each unit at once) warps 0 and 1 meanwhile
+        // find the CTA's expand items
+        if (KS == 1 && !have_range && warp < 2) {
             find_range(warp);
         } else if (tid >= 64 && tid < 64 + TM) {
             const int t = tid - 64;
@@ -529,7 +574,7 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                                      : residual_row(p, pr, p.blk_res[(int64_t)b * S_MAX + (t - rc)], false);
             }
         }
-        have_range = true;
+        have_range = have_range || KS == 1;
         __syncthreads();
 
         // stage geometry: A = the factor stack (the 128-row UMMA M operand; rows
@@ -694,6 +739,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
     //              rows), then the epilogue: TMEM lanes 32 (w % 4) .. + 31
     //              (one token row a thread), the item's 64 columns: + staged
     //              y, one rounding, store; then "acc empty" and "empty".
+    //              In a run that fits the ring the epilogue writes the
+    //              results back into the stage and the producers, whose loads
+    //              are all issued, store them.
     // The producers do not wait for V: y and B do not depend on it, so the
     // first items stream in while the splits are reduced.
     uint8_t *vs = ring + RING_BYTES - VT_BYTES;  // V_ext: two K-major tiles (K 0..63, 64..127)
@@ -752,6 +800,9 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
         const int m_rows = ((M + 15) >> 4) << 4;
         const int bst = (m_rows + S_pad) * 128;
         const int nbs = min(B_MAX_STAGES, (RING_BYTES - VT_BYTES) / bst);
+        // a run whose items all fit the ring at once: the producers, idle
+        // after its loads, store its results (see below)
+        const bool pstore = n <= nbs;
 
         // The run's table: written by the producers and the MMA warp,
         // published to the epilogue warps through "table" (the previous run
@@ -791,6 +842,25 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                 const uint32_t gp = g0 + j - nbs;
                 if (!mbar_wait(empty_bar(gp % B_MAX_STAGES), (gp / B_MAX_STAGES) & 1)) ok_all = false;
                 load_item(j);
+            }
+            if (pstore) {
+                // A run that fits the ring: every load is issued, so the
+                // producers store the items' results (written back into their
+                // stages by the epilogue warps) as each stage empties, 8
+                // threads per 128-byte row piece, and the epilogue warps go on
+                // to the next accumulator at once.
+                for (int j = 0; j < n; ++j) {
+                    const uint32_t gp = g0 + j;
+                    if (!mbar_wait(empty_bar(gp % B_MAX_STAGES), (gp / B_MAX_STAGES) & 1)) ok_all = false;
+                    const int n0 = (u0 + j - ubase) * NC;
+                    const uint8_t *ysp = ring + (j % nbs) * bst;
+                    for (int idx = tid; idx < M * 8; idx += PRODUCER_THREADS) {
+                        const int r = idx >> 3, c = idx & 7, col = n0 + c * 8;
+                        if (col < d_out)
+                            *reinterpret_cast<uint4 *>(pr.y + (int64_t)info.erow[r] * d_out + col) =
+                                *reinterpret_cast<const uint4 *>(ysp + swz128(r, c));
+                    }
+                }
             }
             cp_async_wait<0>();
         } else if (warp == PRODUCER_WARPS) {
@@ -876,6 +946,11 @@ __global__ void __launch_bounds__(APPLY_THREADS, 1) salt_apply_kernel(const __gr
                             make_uint4(yv[4 * c], yv[4 * c + 1], yv[4 * c + 2], yv[4 * c + 3]);
                 }
                 __syncwarp();
+                if (pstore) {
+                    // the producers store the item once its stage is empty
+                    if (lane == 0) mbar_arrive_release(empty_bar(slot));
+                    continue;
+                }
                 // ... then the warp's 32 rows go out whole (all reads first)
                 {
                     uint4 vv[8];
