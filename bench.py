@@ -263,8 +263,8 @@ class Step:
     def swap(self, s):
         region = self.wl_mod.config4_region(s % self.N_ID_SETS)
         hs = self.host_sets[s % 2]
-        for i in range(self.wl_mod.C4_REGION):
-            self.salt.salt_residual_load(self.runner.ctx, region + i, hs[i], self.side)
+        n = self.wl_mod.C4_REGION
+        self.salt.salt_residual_load_batch(self.runner.ctx, list(range(region, region + n)), hs[:n], self.side)
 
     def build(self, s):
         dom, slot = self.ids[s % self.N_ID_SETS]

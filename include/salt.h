@@ -286,6 +286,20 @@ void salt_host_free(void *ptr);
 salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob,
                                salt_stream_t side_stream);
 
+/*
+ * salt_residual_load for n residuals at once (the per-step swap of a
+ * serving engine, Section "Multi-Tenant Serving").  slots[n] (distinct) and
+ * host_blobs[n] are host arrays; every blob is checked as in
+ * salt_residual_load before anything is enqueued (an error leaves every
+ * slot as it was).  On side_stream: one wait for the applies enqueued so
+ * far on every segments object that refers to any of the slots, then one
+ * cudaMemcpyAsync per blob, each followed by its slot's ready event.  The
+ * result is that of n salt_residual_load calls in order; the host-side cost
+ * is one hazard wait instead of n.  n == 0 does nothing.
+ */
+salt_status salt_residual_load_batch(salt_ctx *ctx, int32_t n, const int32_t *slots, const void *const *host_blobs,
+                                     salt_stream_t side_stream);
+
 /* Allocate a segments object able to hold max_tokens tokens of this
  * context (device metadata plus a pinned id staging area).  Synchronous. */
 salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out);

@@ -302,6 +302,70 @@ int64_t thp_bytes()
 std::mutex g_host_mu;
 std::map<void *, size_t> g_host_maps;  // salt_host_alloc regions and their mapped sizes
 
+// Whether [p, p + bytes) lies in one salt_host_alloc region (page-locked by
+// this library: no driver query needed).
+bool in_host_region(const void *p, uint64_t bytes)
+{
+    std::lock_guard<std::mutex> lock(g_host_mu);
+    auto it = g_host_maps.upper_bound(const_cast<void *>(p));
+    if (it == g_host_maps.begin()) return false;
+    --it;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(it->first), q = reinterpret_cast<uintptr_t>(p);
+    return q >= a && q + bytes <= a + it->second;
+}
+
+// Checks of one residual blob for a load into `slot`; *rank and *bytes get
+// its rank and its size (header and payload).
+salt_status check_blob(salt_ctx *ctx, int32_t slot, const void *host_blob, int32_t *rank, uint64_t *bytes)
+{
+    if (slot < 0 || slot >= ctx->n_slots) return fail(ctx, SALT_ERR_SLOT_RANGE, "slot %d outside [0, %d)", slot, ctx->n_slots);
+    if (!host_blob) return fail(ctx, SALT_ERR_INVALID_ARG, "null blob");
+    if (!in_host_region(host_blob, SALT_BLOB_HEADER_BYTES)) {
+        cudaPointerAttributes attr;
+        if (cudaPointerGetAttributes(&attr, host_blob) != cudaSuccess) {
+            cudaGetLastError();
+            return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob pointer is not registered with CUDA");
+        }
+        if (attr.type != cudaMemoryTypeHost)
+            return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob is not page-locked host memory (type %d)", (int)attr.type);
+    }
+    salt_blob_header h;
+    std::memcpy(&h, host_blob, sizeof h);
+    if (h.magic != SALT_BLOB_MAGIC || h.version != 1) return fail(ctx, SALT_ERR_BAD_BLOB, "bad blob magic or version");
+    if (h.n_layers != ctx->n_layers || h.layout_hash != ctx->layout_hash)
+        return fail(ctx, SALT_ERR_BAD_BLOB, "blob was built for another layer table");
+    if (h.rank < 1 || h.rank > ctx->r_max) return fail(ctx, SALT_ERR_RANK, "blob rank %d outside [1, %d]", h.rank, ctx->r_max);
+    uint64_t pay = (uint64_t)(ctx->sum_din + ctx->sum_dout) * (uint64_t)h.rank * 2;
+    if (h.payload_bytes != pay) return fail(ctx, SALT_ERR_BAD_BLOB, "blob payload size mismatch");
+    *rank = h.rank;
+    *bytes = SALT_BLOB_HEADER_BYTES + pay;
+    return SALT_OK;
+}
+
+// The loads of n checked blobs on `side`: readers first (every segments
+// object that names one of the slots waits for its uses, once), then one
+// copy and one ready event per slot.
+salt_status enqueue_loads(salt_ctx *ctx, int32_t n, const int32_t *slots, const void *const *blobs, const int32_t *ranks,
+                          const uint64_t *bytes, cudaStream_t side)
+{
+    for (salt_segments *seg : ctx->segs) {
+        if (!seg->built) continue;
+        bool names = seg->device_ids;
+        for (int32_t i = 0; i < n && !names; ++i) names = seg->refs[slots[i]] != 0;
+        if (!names) continue;
+        seg->stale = true;
+        CUDA_OR_FAIL(ctx, wait_for_uses(seg, side));
+    }
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t slot = slots[i];
+        uint8_t *dst = ctx->pool + (int64_t)slot * ctx->slot_stride;
+        CUDA_OR_FAIL(ctx, cudaMemcpyAsync(dst, blobs[i], bytes[i], cudaMemcpyHostToDevice, side));
+        CUDA_OR_FAIL(ctx, cudaEventRecord(ctx->slot_ready[slot], side));
+        ctx->slot_rank[slot] = ranks[i];
+        ctx->slot_seq[slot] += 1;
+    }
+    return SALT_OK;
+}
 }  // namespace
 
 extern "C" {
@@ -749,39 +813,28 @@ salt_status salt_residual_blob_concat(const salt_config *config, int32_t rc, con
 salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob, salt_stream_t side_stream)
 {
     if (!ctx) return SALT_ERR_INVALID_ARG;
-    if (slot < 0 || slot >= ctx->n_slots) return fail(ctx, SALT_ERR_SLOT_RANGE, "slot %d outside [0, %d)", slot, ctx->n_slots);
-    if (!host_blob) return fail(ctx, SALT_ERR_INVALID_ARG, "null blob");
+    int32_t rank = 0;
+    uint64_t bytes = 0;
+    salt_status st = check_blob(ctx, slot, host_blob, &rank, &bytes);
+    if (st != SALT_OK) return st;
     if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
-    cudaPointerAttributes attr;
-    if (cudaPointerGetAttributes(&attr, host_blob) != cudaSuccess) {
-        cudaGetLastError();
-        return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob pointer is not registered with CUDA");
-    }
-    if (attr.type != cudaMemoryTypeHost)
-        return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob is not page-locked host memory (type %d)", (int)attr.type);
-    salt_blob_header h;
-    std::memcpy(&h, host_blob, sizeof h);
-    if (h.magic != SALT_BLOB_MAGIC || h.version != 1) return fail(ctx, SALT_ERR_BAD_BLOB, "bad blob magic or version");
-    if (h.n_layers != ctx->n_layers || h.layout_hash != ctx->layout_hash)
-        return fail(ctx, SALT_ERR_BAD_BLOB, "blob was built for another layer table");
-    if (h.rank < 1 || h.rank > ctx->r_max) return fail(ctx, SALT_ERR_RANK, "blob rank %d outside [1, %d]", h.rank, ctx->r_max);
-    uint64_t pay = (uint64_t)(ctx->sum_din + ctx->sum_dout) * (uint64_t)h.rank * 2;
-    if (h.payload_bytes != pay) return fail(ctx, SALT_ERR_BAD_BLOB, "blob payload size mismatch");
-    cudaStream_t side = static_cast<cudaStream_t>(side_stream);
+    return enqueue_loads(ctx, 1, &slot, &host_blob, &rank, &bytes, static_cast<cudaStream_t>(side_stream));
+}
 
-    // Readers first: every segments object that names this slot waits for its uses.
-    for (salt_segments *seg : ctx->segs) {
-        if (!seg->built) continue;
-        if (!seg->device_ids && !seg->refs[slot]) continue;
-        seg->stale = true;
-        CUDA_OR_FAIL(ctx, wait_for_uses(seg, side));
+salt_status salt_residual_load_batch(salt_ctx *ctx, int32_t n, const int32_t *slots, const void *const *host_blobs,
+                                     salt_stream_t side_stream)
+{
+    if (!ctx) return SALT_ERR_INVALID_ARG;
+    if (n < 0 || (n > 0 && (!slots || !host_blobs))) return fail(ctx, SALT_ERR_INVALID_ARG, "bad batch of %d loads", n);
+    if (n == 0) return SALT_OK;
+    std::vector<int32_t> ranks(n);
+    std::vector<uint64_t> bytes(n);
+    for (int32_t i = 0; i < n; ++i) {
+        salt_status st = check_blob(ctx, slots[i], host_blobs[i], &ranks[i], &bytes[i]);
+        if (st != SALT_OK) return st;
     }
-    uint8_t *dst = ctx->pool + (int64_t)slot * ctx->slot_stride;
-    CUDA_OR_FAIL(ctx, cudaMemcpyAsync(dst, host_blob, SALT_BLOB_HEADER_BYTES + pay, cudaMemcpyHostToDevice, side));
-    CUDA_OR_FAIL(ctx, cudaEventRecord(ctx->slot_ready[slot], side));
-    ctx->slot_rank[slot] = h.rank;
-    ctx->slot_seq[slot] += 1;
-    return SALT_OK;
+    if (!set_device(ctx)) return fail(ctx, SALT_ERR_CUDA, "cannot select device %d", ctx->device);
+    return enqueue_loads(ctx, n, slots, host_blobs, ranks.data(), bytes.data(), static_cast<cudaStream_t>(side_stream));
 }
 
 salt_status salt_segments_create(salt_ctx *ctx, salt_segments **out)

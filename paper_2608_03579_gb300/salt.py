@@ -79,6 +79,7 @@ _SIGS = {
     "salt_residual_blob_bytes": (_i64, [ctypes.POINTER(salt_config), _i32]),
     "salt_residual_blob_pack": (ctypes.c_int, [ctypes.POINTER(salt_config), _i32, _f32, _vp, _vp, _vp, _i64]),
     "salt_residual_load": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
+    "salt_residual_load_batch": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
     "salt_segments_create": (ctypes.c_int, [_vp, ctypes.POINTER(_vp)]),
     "salt_segments_destroy": (None, [_vp]),
     "salt_build_segments": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp]),
@@ -299,6 +300,16 @@ def salt_host_free(buf) -> None:
 
 def salt_residual_load(ctx, slot: int, host_blob, stream=None) -> None:
     _check(_lib.salt_residual_load(ctx, slot, _ptr(host_blob), _stream(stream)), ctx)
+
+
+def salt_residual_load_batch(ctx, slots, host_blobs, stream=None) -> None:
+    """The loads of salt_residual_load for each (slot, blob) pair, in one call."""
+    n = len(slots)
+    if len(host_blobs) != n:
+        raise ValueError("one blob per slot")
+    sl = (_i32 * max(n, 1))(*[int(x) for x in slots])
+    bl = (_vp * max(n, 1))(*[_ptr(b) for b in host_blobs])
+    _check(_lib.salt_residual_load_batch(ctx, n, sl, bl, _stream(stream)), ctx)
 
 
 def salt_segments_create(ctx) -> int:

@@ -146,3 +146,52 @@ def test_huge_page_host_blob_swap(salt_lib, oracle_mod, wl):
         finally:
             hb.close()
     assert_close(got, _oracle(oracle_mod, w, lambda u: 5 if u == 2 else 0), "huge-page host blob")
+
+
+def test_batch_load_between_batches_on_side_stream(salt_lib, oracle_mod, wl):
+    """salt_residual_load_batch: the same ordering as single loads (the swap
+    waits for the applies that read the slots, the segments turn stale, a
+    rebuild waits for the copies), one call for several slots; a bad blob in
+    the batch loads nothing."""
+    from paper_2608_03579_gb300.runner import SaltRunner, bf16_bits, bf16_tensor
+    salt = salt_lib
+    w = _workload(wl)
+    side = torch.cuda.Stream()
+    comp = torch.cuda.Stream()
+    with SaltRunner(w) as r:
+        r.pin_centroids()
+        r.load_slots()
+        x = bf16_tensor(w.x(0))
+        y1 = bf16_tensor(w.y_in(0))
+        y2 = bf16_tensor(w.y_in(0))
+        y3 = bf16_tensor(w.y_in(0))
+        r.build(stream=comp)
+        salt.salt_lora_apply(r.ctx, r.seg, 0, x, y1, comp)
+        # one blob from a huge-page region of the library, two from torch's pinned memory
+        nb = r.blob_bytes(2)
+        region = salt.salt_host_alloc(nb)
+        try:
+            b0 = r.make_blob(0, version=5, out=region.tensor[:nb])
+            b2 = r.make_blob(2, version=5)
+            b5 = r.make_blob(5, version=5)
+            # a batch holding one bad blob is refused before anything is enqueued
+            bad = r.make_blob(4, version=5).clone().pin_memory()
+            bad[0] ^= 0xFF  # magic
+            with pytest.raises(salt.SaltError):
+                salt.salt_residual_load_batch(r.ctx, [0, 4], [b0, bad], side)
+            salt.salt_lora_apply(r.ctx, r.seg, 0, x, y2, comp)  # still valid: nothing was loaded
+            salt.salt_residual_load_batch(r.ctx, [0, 2, 5], [b0, b2, b5], side)
+            with pytest.raises(salt.SaltError) as e:
+                salt.salt_lora_apply(r.ctx, r.seg, 0, x, y3, comp)
+            assert e.value.name == "SALT_ERR_STALE_SEGMENTS"
+            r.build(stream=comp)
+            salt.salt_lora_apply(r.ctx, r.seg, 0, x, y3, comp)
+            torch.cuda.synchronize()
+            assert r.device_error() == 0
+            got1, got2, got3 = bf16_bits(y1), bf16_bits(y2), bf16_bits(y3)
+        finally:
+            torch.cuda.synchronize()
+            salt.salt_host_free(region)
+    assert_close(got1, _oracle(oracle_mod, w, lambda u: 0), "before the batch")
+    assert_close(got2, _oracle(oracle_mod, w, lambda u: 0), "after the refused batch")
+    assert_close(got3, _oracle(oracle_mod, w, lambda u: 5 if u in (0, 2, 5) else 0), "after the batch")
