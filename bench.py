@@ -224,6 +224,7 @@ class Step:
         pitch = (nb + 255) // 256 * 256
         n_host = 64 if rank16 else 2 * wl.C4_REGION
         self.host_buf = salt.salt_host_alloc(n_host * pitch)
+        self.host_huge = huge_page_bytes(self.host_buf.ptr)
         blob_at = lambda k: self.host_buf.tensor[k * pitch:k * pitch + nb]
         if rank16:
             base = [r.make_blob(u, 0, r_slot, out=blob_at(u)) for u in range(64)]
@@ -483,6 +484,25 @@ def run_reference(args, rank, world, pg):
                              "cores_source": "os.sched_getaffinity"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def huge_page_bytes(ptr: int):
+    """(mapping bytes, bytes backed by transparent huge pages) of the process
+    mapping that holds `ptr`, from /proc/self/smaps; (None, None) if unknown."""
+    try:
+        cur = None
+        with open("/proc/self/smaps") as f:
+            for line in f:
+                head = line.split(" ", 1)[0]
+                if "-" in head and ":" not in head:
+                    a, b = (int(x, 16) for x in head.split("-"))
+                    cur = [b - a, None] if a <= ptr < b else None
+                elif cur is not None and line.startswith("AnonHugePages:"):
+                    cur[1] = int(line.split()[1]) * 1024
+                    return cur[0], cur[1]
+    except (OSError, ValueError):
+        pass
+    return None, None
 
 
 def traffic_from_profile():
@@ -754,6 +774,7 @@ def run_salt(args, rank, world, local, pg):
                 "gpu_launches": args.steps * (n_launch + 1),
                 "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
                 "swap_ms_per_step_alone": swap_ms, "apply_only_ms_per_step": apply_only_ms,
+                "swap_host_memory": dict(zip(("bytes", "huge_page_bytes"), st.host_huge)),
                 "apply_kernel_by_group": per_kind,
                 "apply_launch_shape": {k: ctx_info[k] for k in ("apply_ctas", "k_splits_max", "apply_smem_bytes",
                                                                   "block_tokens", "block_users")},

@@ -258,8 +258,9 @@ void salt_fold_plan_destroy(salt_fold_plan *plan);
 /*
  * Page-locked host memory for residual blobs, backed by transparent huge
  * pages where the kernel offers them (anonymous mapping rounded up to the
- * huge-page size, madvise(MADV_HUGEPAGE), every page touched, then
- * cudaHostRegister).  The host-to-device copies of a swap translate host
+ * huge-page size, madvise(MADV_HUGEPAGE), every page touched, a request to
+ * collapse what still has base pages (MADV_COLLAPSE, where the kernel has
+ * it), then cudaHostRegister).  The host-to-device copies of a swap translate host
  * addresses page by page; with the base pages of an ordinary pinned
  * allocation (64 KiB on Arm servers) sustained swapping was measured to
  * stall for 30-100 ms every few hundred copies, with huge pages not at all.

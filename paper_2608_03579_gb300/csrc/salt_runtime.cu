@@ -320,7 +320,7 @@ salt_status check_blob(salt_ctx *ctx, int32_t slot, const void *host_blob, int32
 {
     if (slot < 0 || slot >= ctx->n_slots) return fail(ctx, SALT_ERR_SLOT_RANGE, "slot %d outside [0, %d)", slot, ctx->n_slots);
     if (!host_blob) return fail(ctx, SALT_ERR_INVALID_ARG, "null blob");
-    if (!in_host_region(host_blob, SALT_BLOB_HEADER_BYTES)) {
+    auto pinned_by_driver = [&]() -> salt_status {
         cudaPointerAttributes attr;
         if (cudaPointerGetAttributes(&attr, host_blob) != cudaSuccess) {
             cudaGetLastError();
@@ -328,6 +328,13 @@ salt_status check_blob(salt_ctx *ctx, int32_t slot, const void *host_blob, int32
         }
         if (attr.type != cudaMemoryTypeHost)
             return fail(ctx, SALT_ERR_NOT_PINNED_HOST, "blob is not page-locked host memory (type %d)", (int)attr.type);
+        return SALT_OK;
+    };
+    // the header is read on the host only once it is known to be host memory
+    const bool in_region = in_host_region(host_blob, SALT_BLOB_HEADER_BYTES);
+    if (!in_region) {
+        salt_status st = pinned_by_driver();
+        if (st != SALT_OK) return st;
     }
     salt_blob_header h;
     std::memcpy(&h, host_blob, sizeof h);
@@ -337,6 +344,10 @@ salt_status check_blob(salt_ctx *ctx, int32_t slot, const void *host_blob, int32
     if (h.rank < 1 || h.rank > ctx->r_max) return fail(ctx, SALT_ERR_RANK, "blob rank %d outside [1, %d]", h.rank, ctx->r_max);
     uint64_t pay = (uint64_t)(ctx->sum_din + ctx->sum_dout) * (uint64_t)h.rank * 2;
     if (h.payload_bytes != pay) return fail(ctx, SALT_ERR_BAD_BLOB, "blob payload size mismatch");
+    if (in_region && !in_host_region(host_blob, SALT_BLOB_HEADER_BYTES + pay)) {
+        salt_status st = pinned_by_driver();  // the blob runs past the region
+        if (st != SALT_OK) return st;
+    }
     *rank = h.rank;
     *bytes = SALT_BLOB_HEADER_BYTES + pay;
     return SALT_OK;
@@ -381,6 +392,11 @@ void *salt_host_alloc(int64_t bytes)
     madvise(p, size, MADV_HUGEPAGE);  // advice only: base pages if refused
 #endif
     std::memset(p, 0, size);  // fault every page in before it is registered
+    // Where the faults got base pages (no free huge page at the time),
+    // ask the kernel to collapse the range into huge pages now (Linux 6.1
+    // and later; refused or ignored elsewhere, which leaves base pages).
+    constexpr int kMadvCollapse = 25;
+    madvise(p, size, kMadvCollapse);
     if (cudaHostRegister(p, size, cudaHostRegisterDefault) != cudaSuccess) {
         cudaGetLastError();
         munmap(p, size);

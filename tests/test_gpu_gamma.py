@@ -57,6 +57,21 @@ def _check(salt, ctx, seg, oracle_mod, dom, slot, gb):
         covered[s0:s0 + n] += 1
     active = (dom[ref["perm"]] >= 0) | (slot[ref["perm"]] >= 0)
     np.testing.assert_array_equal(covered, active.astype(int))
+    # The blocks index the apply order: the same tokens stably sorted by
+    # (domain, slot, bin), so that a user's tokens in several bins are one
+    # run of its block and a block holds at most umax distinct users (here
+    # (128 - 16) / 2 = 56), however many bins they span.
+    dom, slot, gb = (np.asarray(a) for a in (dom, slot, gb))
+    gbk = np.where(dom >= 0, gb, -1)
+    apply_order = np.lexsort((np.arange(len(dom)), gbk, slot, dom))
+    for (s0, n, d) in got["blocks"]:
+        toks = apply_order[s0:s0 + n]
+        assert (dom[toks] == d).all()
+        sl = slot[toks]
+        users = np.unique(sl[sl >= 0])
+        assert len(users) <= (TM - 16) // 2
+        runs = 1 + int(np.count_nonzero(np.diff(sl)))  # every user's tokens are contiguous
+        assert runs == len(np.unique(sl))
 
 
 @pytest.mark.parametrize("T", [1, 77, 512, 4096, 16384])
