@@ -20,6 +20,8 @@
 
 #include <sys/mman.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "salt_internal.cuh"
 
 using namespace salt;
@@ -91,6 +93,16 @@ struct salt_host_pipe {
 };
 
 namespace {
+
+// A named NVTX range around a library call on the host (what a timeline
+// tool shows next to the kernels the call enqueues); free when no tool is
+// attached.
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
+};
 
 salt_status fail(salt_ctx *ctx, salt_status s, const char *fmt, ...)
 {
@@ -572,6 +584,7 @@ void salt_ctx_destroy(salt_ctx *ctx)
 salt_status salt_centroid_pin(salt_ctx *ctx, int32_t domain, int32_t rc, const void *At_c, const void *B_c,
                               float s_c)
 {
+    NvtxRange nvtx_range("salt_centroid_pin");
     if (!ctx) return SALT_ERR_INVALID_ARG;
     if (domain < 0 || domain >= ctx->n_domains)
         return fail(ctx, SALT_ERR_DOMAIN_RANGE, "domain %d outside [0, %d)", domain, ctx->n_domains);
@@ -642,6 +655,7 @@ salt_status salt_residual_blob_pack(const salt_config *config, int32_t rank, flo
 salt_status salt_centroid_fold(salt_ctx *ctx, int32_t domain, int32_t layer, float gamma, void *W, int32_t layout,
                                salt_stream_t stream)
 {
+    NvtxRange nvtx_range("salt_centroid_fold");
     if (!ctx) return SALT_ERR_INVALID_ARG;
     if (domain < 0 || domain >= ctx->n_domains)
         return fail(ctx, SALT_ERR_DOMAIN_RANGE, "domain %d outside [0, %d)", domain, ctx->n_domains);
@@ -732,6 +746,7 @@ salt_status salt_fold_plan_create(salt_ctx *ctx, int32_t domain, int32_t n, cons
 
 salt_status salt_fold_plan_run(salt_fold_plan *plan, float gamma, salt_stream_t stream)
 {
+    NvtxRange nvtx_range("salt_fold_plan_run");
     if (!plan || !plan->ctx) return SALT_ERR_INVALID_ARG;
     salt_ctx *ctx = plan->ctx;
     if (ctx->dom_rc[plan->domain] != plan->rc)
@@ -755,6 +770,7 @@ void salt_fold_plan_destroy(salt_fold_plan *plan)
 salt_status salt_align_loss(int32_t n, const salt_align_pair *pairs, float eps, float *loss, float *cosine,
                             salt_stream_t stream)
 {
+    NvtxRange nvtx_range("salt_align_loss");
     return align_loss_run(n, pairs, eps, loss, cosine, static_cast<cudaStream_t>(stream));
 }
 
@@ -828,6 +844,7 @@ salt_status salt_residual_blob_concat(const salt_config *config, int32_t rc, con
 
 salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blob, salt_stream_t side_stream)
 {
+    NvtxRange nvtx_range("salt_residual_load");
     if (!ctx) return SALT_ERR_INVALID_ARG;
     int32_t rank = 0;
     uint64_t bytes = 0;
@@ -840,6 +857,7 @@ salt_status salt_residual_load(salt_ctx *ctx, int32_t slot, const void *host_blo
 salt_status salt_residual_load_batch(salt_ctx *ctx, int32_t n, const int32_t *slots, const void *const *host_blobs,
                                      salt_stream_t side_stream)
 {
+    NvtxRange nvtx_range("salt_residual_load_batch");
     if (!ctx) return SALT_ERR_INVALID_ARG;
     if (n < 0 || (n > 0 && (!slots || !host_blobs))) return fail(ctx, SALT_ERR_INVALID_ARG, "bad batch of %d loads", n);
     if (n == 0) return SALT_OK;
@@ -946,6 +964,7 @@ salt_status salt_build_segments_gamma(salt_ctx *ctx, salt_segments *seg, const i
                                       const int32_t *gamma_bins, const int32_t *slot_ids, int32_t n_tokens,
                                       int32_t n_gamma, const float *gamma, salt_stream_t stream_)
 {
+    NvtxRange nvtx_range("salt_build_segments");
     if (!ctx || !seg || seg->ctx != ctx) return SALT_ERR_INVALID_ARG;
     if (n_tokens < 0) return fail(ctx, SALT_ERR_INVALID_ARG, "negative token count");
     if (n_tokens > ctx->max_tokens)
@@ -1107,6 +1126,7 @@ namespace {
 salt_status apply_grouped(salt_ctx *ctx, const salt_segments *seg_, int32_t n, const int32_t *layers,
                           const void *const *x, void *const *y, salt_stream_t stream_, bool shrink_only)
 {
+    NvtxRange nvtx_range("salt_lora_apply");
     if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
     salt_segments *seg = const_cast<salt_segments *>(seg_);
     if (n < 1 || n > SALT_MAX_GROUP || !layers || !x || !y)
@@ -1181,6 +1201,7 @@ salt_status salt_lora_apply_grouped(salt_ctx *ctx, const salt_segments *seg, int
 salt_status salt_lora_apply_with_base(salt_ctx *ctx, const salt_segments *seg_, int32_t layer, const void *x,
                                       const void *W, int32_t layout, void *y, salt_stream_t stream_)
 {
+    NvtxRange nvtx_range("salt_lora_apply_with_base");
     if (!ctx || !seg_ || seg_->ctx != ctx) return SALT_ERR_INVALID_ARG;
     salt_segments *seg = const_cast<salt_segments *>(seg_);
     if (layer < 0 || layer >= ctx->n_layers)
@@ -1359,6 +1380,7 @@ void salt_host_pipe_destroy(salt_host_pipe *pipe)
 salt_status salt_lora_apply_host(salt_host_pipe *pipe, const salt_segments *seg, int32_t n, const int32_t *layers,
                                  const void *const *x_host, void *const *y_host, salt_stream_t stream_)
 {
+    NvtxRange nvtx_range("salt_lora_apply_host");
     if (!pipe || !pipe->ctx) return SALT_ERR_INVALID_ARG;
     salt_ctx *ctx = pipe->ctx;
     if (!seg || seg->ctx != ctx) return fail(ctx, SALT_ERR_INVALID_ARG, "segments of another context");
