@@ -28,3 +28,19 @@ def test_timeout_flag_makes_the_run_invalid():
     assert not d.valid
     s = d.summary()
     assert s["valid"] is False and s["device_error_flags"] == {"timed": "0x20"}
+
+
+def test_huge_page_report_finds_the_mapping():
+    """The swap's host-memory report reads the mapping that holds a pointer
+    from /proc/self/smaps: its size, and the bytes backed by huge pages."""
+    import ctypes
+    import mmap
+    n = 4 << 20
+    m = mmap.mmap(-1, n)
+    buf = (ctypes.c_char * n).from_buffer(m)
+    size, huge = bench.huge_page_bytes(ctypes.addressof(buf))
+    assert size is not None and size >= n
+    assert huge is not None and 0 <= huge <= size
+    del buf
+    m.close()
+    assert bench.huge_page_bytes(0) == (None, None)
